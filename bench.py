@@ -1,0 +1,466 @@
+"""Benchmark of the RhymeFlow asynchronous step core on GB300.
+
+A "step" is one asynchronous denoising step of the trajectory, all four
+library calls (compaction, Eq. 3 projection, active-query attention, Euler
+update) over the workload's synthetic inputs resident in HBM.  Timed step k is
+schedule step s = k mod S, so K = S steps is one whole trajectory.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config small]
+    python bench.py --impl reference ...   # the CPU oracle on the host cores
+
+value        attention TFLOP/s of the whole step core (algorithmic FLOPs
+             4 * active_rows * F*N * d * H summed over the timed steps, divided
+             by the device time of the timed steps), summed over ranks
+roofline     rf_attn alone: its algorithmic FLOPs per launch / its average launch
+             time (CUDA events around each launch on the launching stream)
+e2e          the same metric with every step's inputs copied from pinned host
+             memory and its outputs read back, inside the timed region
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "rf_attn TFLOP/s (% BF16 peak); step-core ms vs all-frames-active on 1 GB300"
+UNIT = "TFLOP/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# DRAM traffic of rf_attn measured with ncu (dram__bytes_read.sum + dram__bytes_write.sum),
+# per launch averaged over one trajectory of the "small" workload, valid only for the kernel
+# source with this hash.
+ATTN_TRAFFIC = {"sha256_rf_attn_cu": None, "workload": "small", "bytes_per_launch": None}
+
+
+def _env_rank():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def _sha(path):
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) != 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for _, _, flags in rows for n, fl in zip(names, flags)
+                          if fl.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+def _gpu_index(local_rank):
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [x.strip() for x in vis.split(",")]
+        if local_rank < len(ids) and ids[local_rank].isdigit():
+            return int(ids[local_rank])
+    return local_rank
+
+
+# ---------------------------------------------------------------------------
+# The GPU arm
+# ---------------------------------------------------------------------------
+def run_gpu(args):
+    import torch
+    import workloads as wl
+    import paper_2606_06309_gb300 as rf
+    from paper_2606_06309_gb300.stepcore import StepCore, upload_plan
+
+    rank, world, local = _env_rank()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    rf.load()
+    dev = torch.device("cuda", local)
+    w = wl.get(args.config)
+    E = w.N * w.C
+    S = w.S
+    plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, dev)
+    core = StepCore(w.F, w.N, E, w.H, w.d, plan, dev)
+    core.set_state(wl.latents(w, device=dev))
+    Q, K, V = wl.qkv(w, device=dev)
+    O = torch.empty_like(Q)
+    vel = [wl.velocity(w, s, device=dev) for s in range(S)]
+    stream = torch.cuda.current_stream(dev)
+    mask_host = plan.host["mask"]
+    A_per_step = mask_host.sum(axis=1)
+    flops_step = [4 * int(A_per_step[s]) * w.N * w.S_tok * w.d * w.H for s in range(S)]
+
+    # all-frames-active comparison plan (mask = 1, every frame one step)
+    plan_all = upload_plan(w.F, w.S, [1] * w.F, [1] * S, 0, dev)
+    core_all = StepCore(w.F, w.N, E, w.H, w.d, plan_all, dev)
+    core_all.set_state(wl.latents(w, device=dev))
+    flops_all = 4 * w.F * w.N * w.S_tok * w.d * w.H
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+            torch.cuda.synchronize()
+
+    def timed(c, K_steps, W_steps, per_launch=False):
+        for k in range(W_steps):
+            c.run(k % S, vel[k % S], O, Q, K, V, w.softmax_scale)
+        barrier()
+        ev = [] if per_launch else None
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for k in range(K_steps):
+            s = k % S
+            c.compact(s)
+            c.project(s)
+            if per_launch:
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                c.attn(O, Q, K, V, w.softmax_scale)
+                b.record(stream)
+                ev.append((s, a, b))
+            else:
+                c.attn(O, Q, K, V, w.softmax_scale)
+            c.step(s, vel[s])
+        t1.record(stream)
+        barrier()
+        ms = t0.elapsed_time(t1)
+        return ms, ev
+
+    K_steps, W_steps = args.steps, args.warmup
+    with ClockSampler(_gpu_index(local)) as clk:
+        ms, _ = timed(core, K_steps, W_steps)
+    clocks = clk.summary()
+    # max over ranks
+    ms_t = torch.tensor([ms], device=dev, dtype=torch.float64)
+    if dist is not None:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms = float(ms_t.item())
+    total_flops = sum(flops_step[k % S] for k in range(K_steps)) * world
+    value = total_flops / (ms * 1e-3) / 1e12
+
+    # per-launch attention timing for the roofline (separate pass, same work)
+    _, ev = timed(core, K_steps, 0, per_launch=True)
+    launch_ms = [a.elapsed_time(b) for _, a, b in ev]
+    attn_ms_total = sum(launch_ms)
+    attn_flops_total = sum(flops_step[s] for s, _, _ in ev)
+    achieved = attn_flops_total / (attn_ms_total * 1e-3) / 1e12
+    per_launch_flops = attn_flops_total / len(ev)
+    # all-frames-active comparison, same number of steps
+    ms_all, _ = timed(core_all, K_steps, min(W_steps, 3))
+
+    # end to end through the public API with host buffers
+    e2e = run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist, world)
+
+    peaks, peak_src = _peaks()
+    traffic = None
+    attn_src = os.path.join(ROOT, "paper_2606_06309_gb300", "csrc", "rf_attn.cu")
+    if ATTN_TRAFFIC["sha256_rf_attn_cu"] == _sha(attn_src) and args.config == ATTN_TRAFFIC["workload"]:
+        traffic = ATTN_TRAFFIC["bytes_per_launch"]
+    bw = run_bandwidth(w, dev, peaks) if not args.no_bandwidth else None
+    status = int(core.status.item()) | int(core_all.status.item())
+
+    out = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": K_steps, "warmup": W_steps, "ms_per_step": round(ms / K_steps, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads x {w.d}, "
+                        f"latent {w.C} ch, {w.S} flow-matching steps",
+            "keyframes": list(w.keyframes), "stride": f"{w.stride[0]}..{w.stride[-1]}",
+            "active_frames_per_step_avg": float(A_per_step.mean()),
+            "l2": f"inputs larger than L2: Q/K/V {3 * Q.numel() * 2 / 1e6:.0f} MB",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "peak_source": peak_src,
+        },
+        "step_core_ms": round(ms / K_steps, 5),
+        "step_core_ms_all_active": round(ms_all / K_steps, 5),
+        "speedup_vs_all_active": round(ms_all / ms, 4),
+        "ideal_speedup_vs_all_active": round(K_steps * flops_all /
+                                             sum(flops_step[k % S] for k in range(K_steps)), 4),
+        "roofline": {
+            "bound": "tensor", "kernel": "rf_attn", "achieved": round(achieved, 2),
+            "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+            "frac": round(achieved / peaks["bf16_tflops"], 4),
+            "frac_of_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4),
+            "traffic": traffic,
+            "flops_per_launch": per_launch_flops,
+            "avg_launch_ms": round(attn_ms_total / len(ev), 5),
+        },
+        "bandwidth_kernels": bw,
+        "e2e": e2e,
+        "gpu_launches": 4 * K_steps,
+        "clocks": clocks,
+        "device_status": status,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist, world):
+    """Every step: H2D of Q, K, V and the velocity from pinned host memory, the four
+    library calls, D2H of the attention output and the updated latent state."""
+    import torch
+    S = w.S
+    hQ, hK, hV = (x.cpu().pin_memory() for x in (Q, K, V))
+    hv = [v.cpu().pin_memory() for v in vel]
+    hO = torch.empty(Q.shape, dtype=Q.dtype).pin_memory()
+    hz = torch.empty(core.z2.shape, dtype=core.z2.dtype).pin_memory()
+    dQ, dK, dV = (torch.empty_like(x) for x in (Q, K, V))
+    dv = torch.empty_like(vel[0])
+    dO = torch.empty_like(Q)
+    K_steps = max(1, min(args.steps, args.e2e_steps))
+
+    def one(k):
+        s = k % S
+        dQ.copy_(hQ, non_blocking=True)
+        dK.copy_(hK, non_blocking=True)
+        dV.copy_(hV, non_blocking=True)
+        dv.copy_(hv[s], non_blocking=True)
+        core.run(s, dv, dO, dQ, dK, dV, w.softmax_scale)
+        hO.copy_(dO, non_blocking=True)
+        hz.copy_(core.z2, non_blocking=True)
+
+    for k in range(3):
+        one(k)
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(K_steps):
+        one(k)
+    t1.record(stream)
+    barrier()
+    ms = t0.elapsed_time(t1)
+    ms_t = torch.tensor([ms], device=Q.device, dtype=torch.float64)
+    if dist is not None:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms = float(ms_t.item())
+    flops = sum(flops_step[k % S] for k in range(K_steps)) * world
+    h2d = 3 * Q.numel() * Q.element_size() + vel[0].numel() * 4
+    d2h = Q.numel() * Q.element_size() + core.z2.numel() * 4
+    return {"value": round(flops / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "steps": K_steps,
+            "ms_per_step": round(ms / K_steps, 5), "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h}
+
+
+def run_bandwidth(w, dev, peaks):
+    """rf_project and rf_step at the hidden-width stress shape (C = H*d fp32, the width of
+    the per-layer rolling cache), L2 flushed before every launch."""
+    import torch
+    import workloads as wl
+    import paper_2606_06309_gb300 as rf
+    F, E = w.F, w.N * w.H * w.d
+    mem = (2 * F * E + 2 * F * E) * 4
+    if mem > 0.5 * torch.cuda.get_device_properties(dev).total_memory:
+        return None
+    z2 = torch.empty(2, F, E, device=dev)
+    z2[0].copy_(wl.hidden_latents(w, 0, device=dev))
+    z2[1].copy_(wl.hidden_latents(w, 1, device=dev))
+    ctx = torch.empty(F, E, device=dev)
+    v = wl.hidden_latents(w, 2, device=dev)
+    p = rf.rf_plan_build(w.F, w.S, w.is_key, w.stride, w.T_w)
+    s = 1 if w.S > 1 else 0  # a step with skipped frames
+    mask = torch.from_numpy(p["mask"][s]).to(dev)
+    alpha = torch.from_numpy(p["alpha"][s]).to(dev)
+    beta = torch.from_numpy(p["beta"][s]).to(dev)
+    slot = torch.from_numpy(p["cur_slot"][s]).to(dev)
+    dt = torch.from_numpy(p["dt"][s]).to(dev)
+    act = torch.zeros(F, dtype=torch.int32, device=dev)
+    skp = torch.zeros(F, dtype=torch.int32, device=dev)
+    cnt = torch.zeros(2, dtype=torch.int32, device=dev)
+    rf.rf_schedule_compact(mask, F, w.N, act, skp, None, cnt)
+    flush = torch.empty(256 * 1024 * 1024 // 4, device=dev)
+    A = int(p["mask"][s].sum())
+    bytes_project = (12 * (F - A) + 8 * A) * E
+    bytes_step = 12 * A * E
+    res = {}
+    for name, fn, nbytes in (
+            ("rf_project", lambda: rf.rf_project(ctx, z2, slot, alpha, beta, F, E), bytes_project),
+            ("rf_step", lambda: rf.rf_step(z2, slot, v, dt, act, cnt, F, E), bytes_step)):
+        times = []
+        for rep in range(13):
+            flush.fill_(rep)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            if rep >= 3:
+                times.append(a.elapsed_time(b))
+        ms = statistics.median(times)
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        res[name] = {"GB/s": round(gbs, 1), "frac": round(gbs / peaks["hbm_gbs"], 4),
+                     "peak": peaks["hbm_gbs"], "ms": round(ms, 4), "bytes": nbytes,
+                     "shape": f"F={F} x E={E} fp32 (C = H*d = {w.H * w.d}), step {s}, A={A}"}
+    del z2, ctx, v, flush
+    torch.cuda.empty_cache()
+    return res
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+def cpu_baseline(w, budget_s=15.0):
+    """The fp64 oracle as it stands, on a bounded sample of one step: schedule,
+    projection and Euler update for every frame at latent width, and attention for a
+    growing number of sampled active query rows (all heads, all keys) until the budget
+    is spent.  Throughput is the sample's algorithmic attention FLOPs per second."""
+    import numpy as np
+    import torch
+    import oracle
+    import workloads as wl
+    Q, K, V = wl.qkv(w)  # host copy of the same seeded inputs
+    plan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+    s = 0
+    mask = plan["mask"][s]
+    rows_all = np.array([f * w.N + p for f in range(w.F) if mask[f] for p in range(w.N)])
+    rng = np.random.default_rng(0)
+    z = wl.latents(w).double().numpy()
+    v = wl.velocity(w, s).double().numpy()
+    t0 = time.perf_counter()
+    oracle.compact(mask, w.N)
+    oracle.project(z, z, plan["alpha"][s])
+    oracle.euler(z, v, plan["dt"][s])
+    n, flops, elapsed = 64, 0, time.perf_counter() - t0
+    while True:
+        rows = rng.choice(rows_all, size=min(n, len(rows_all)), replace=False)
+        t1 = time.perf_counter()
+        oracle.attention(Q, K, V, rows, w.softmax_scale)
+        elapsed += time.perf_counter() - t1
+        flops += oracle.flops_attn(len(rows), w.S_tok, w.d, w.H)
+        if elapsed >= budget_s or n >= len(rows_all):
+            break
+        n *= 2
+    return {"value": round(flops / elapsed / 1e12, 6), "unit": UNIT, "cores": os.cpu_count(),
+            "kind": "oracle", "seconds": round(elapsed, 2),
+            "sample": f"step {s} of {w.name}: full schedule/projection/Euler at latent width "
+                      f"plus attention of sampled active rows x {w.H} heads x {w.S_tok} keys "
+                      f"(fp64 numpy, {flops / 1e12:.3f} TFLOP)"}
+
+
+def run_reference(args):
+    rank, world, _ = _env_rank()
+    if rank != 0:
+        return
+    import workloads as wl
+    w = wl.get(args.config)
+    vals = []
+    budget = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    for k in range(args.warmup + args.steps):
+        cb = cpu_baseline(w, budget_s=budget)
+        if k >= args.warmup:
+            vals.append(cb)
+    value = statistics.mean(c["value"] for c in vals)
+    secs = sum(c["seconds"] for c in vals)
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(1000 * secs / len(vals), 3), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads "
+                                  f"x {w.d}, latent {w.C} ch, {w.S} flow-matching steps"},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
+                            "kind": "oracle", "sample": vals[0]["sample"]},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--config", default="small")
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-bandwidth", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl != "reference":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,188 @@
+/*
+ * rf.h -- C ABI of the RhymeFlow asynchronous denoising step core on GB300.
+ *
+ * RhymeFlow (Sec. 3.2, Algorithm 2) denoises video latent frames on different
+ * schedules: keyframes take one flow-matching step every timestep, non-keyframes
+ * jump n_skip steps at once on their scheduled steps.  At every timestep only
+ * the active frames issue attention queries; they attend to keys and values of
+ * the whole latent sequence, in which the skipped frames are represented by a
+ * linear projection of their latent trajectory (Eq. 3).  Afterwards only the
+ * active frames take their Euler step.
+ *
+ * One step of that core is four calls, all asynchronous on a caller-provided
+ * CUDA stream and all working on caller-owned device buffers:
+ *
+ *   rf_schedule_compact  active-frame mask -> frame / token index lists
+ *   rf_project           Eq. 3 for skipped frames, copy for active frames
+ *   rf_attn              active-query x full-sequence attention (bf16, tcgen05)
+ *   rf_step              Euler update of the active frames
+ *
+ * plus the host planner rf_plan_build that turns a keyframe set and a stride
+ * schedule into the per-step masks and weights.
+ *
+ * Conventions common to every call:
+ *  - Pointers named d_* are device pointers, h_* host pointers.  The caller owns
+ *    every buffer; no call allocates, frees or retains memory beyond its return
+ *    (rf_attn keeps a small per-process cache of device properties only).
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
+ *    enqueued and the call returns; nothing synchronises the host.
+ *  - Errors that the host can see (null pointers, bad sizes, unsupported head
+ *    dim, misalignment) are returned before anything is enqueued.  A failed
+ *    kernel launch returns RF_ERR_CUDA.  Errors found on the device are written
+ *    to the optional device status word of rf_attn and never trap or hang.
+ *  - Frame-major latent layout: a latent state is [F][E] fp32 with E elements
+ *    per frame (E = N*C for N tokens of C channels).  The two-slot store is
+ *    [2][F][E]: slot cur_slot[f] holds frame f's current state and slot
+ *    1-cur_slot[f] the state before its last jump (the "before"/"after" pair of
+ *    Appendix B.2; shift-and-store is a slot flip, not a copy).
+ */
+#ifndef RF_H_
+#define RF_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;
+typedef struct CUstream_st* rf_stream_t; /* == cudaStream_t */
+
+typedef enum {
+  RF_OK = 0,
+  RF_ERR_INVALID_ARG = 1,     /* null pointer, negative or overflowing size */
+  RF_ERR_UNSUPPORTED = 2,     /* e.g. head dim not in {64, 128}, no sm_103 device */
+  RF_ERR_MISALIGNED = 3,      /* pointer or stride breaks a 16-byte TMA rule */
+  RF_ERR_CUDA = 4,            /* a CUDA runtime call or kernel launch failed */
+  RF_ERR_DEVICE_TIMEOUT = 5   /* a bounded device-side wait expired (status word) */
+} rf_status;
+
+/* Human-readable name of a status code.  Never NULL; static storage. */
+const char* rf_status_str(int status);
+
+/* Library ABI version (major*100 + minor). */
+int rf_version(void);
+
+/* Detail of the most recent non-OK status returned to the calling thread (which check
+ * or CUDA call failed, with the CUDA error string), or "" if none.  Thread-local static
+ * storage, valid until the thread's next call into the library. */
+const char* rf_last_error(void);
+
+/*
+ * rf_plan_build -- host planner (CPU, deterministic): Algorithm 2 and Eq. 2.
+ *
+ * Steps s = 0..S-1 run from sigma_0 down to sigma_S = 0 (Algorithm 2's t = T..1).
+ * A frame is active at step s if it is a keyframe, if s < T_w (synchronous
+ * warm-up, Sec. 3.2.1), or if its state has reached step s (its "due" step).
+ * An active keyframe (or any frame in warm-up) advances one step; an active
+ * non-keyframe jumps h_stride[s] steps, the last jump clamped to sigma_S.
+ * Under a constant stride this equals Algorithm 2's modulo rule.
+ *
+ *   F, S        frames, steps (F >= 1, S >= 1, F*S <= 2^31-1)
+ *   h_is_key    [F]   nonzero = keyframe
+ *   h_stride    [S]   skip stride per step, each >= 1
+ *   T_w         warm-up steps, 0 <= T_w <= S
+ *   h_sigma     [S+1] noise levels, strictly decreasing, sigma[S] = 0;
+ *               NULL = uniform sigma_s = 1 - s/S
+ * Outputs (caller-allocated host arrays, all [S][F] row-major):
+ *   h_mask      1 = active at step s
+ *   h_alpha     Eq. 3 weight for skipped frames,
+ *               (sigma_start - sigma_s)/(sigma_start - sigma_due) computed in
+ *               double and rounded to float; 1 for active frames; 0 when
+ *               sigma_start == sigma_due
+ *   h_beta      1 - alpha, computed in double and rounded to float
+ *   h_dt        Euler step sigma_due - sigma_s for active frames, 0 otherwise
+ *   h_cur_slot  slot of the two-slot store holding the frame's current state
+ *               when step s begins (may be NULL)
+ * Returns RF_ERR_INVALID_ARG on bad sizes / null pointers / stride < 1 / bad sigma.
+ */
+rf_status rf_plan_build(int F, int S, const uint8_t* h_is_key, const int32_t* h_stride, int T_w,
+                        const double* h_sigma, uint8_t* h_mask, float* h_alpha, float* h_beta,
+                        float* h_dt, uint8_t* h_cur_slot);
+
+/*
+ * rf_schedule_compact -- Algorithm 2's active set I_active as index lists.
+ *
+ *   d_mask       [F] uint8, nonzero = active
+ *   F, N         frames (1..4096), tokens per frame (>= 1, F*N <= 2^31-1)
+ * Outputs (device, caller-allocated):
+ *   d_active     [F] int32: active frames ascending in [0, A); rest untouched
+ *   d_skipped    [F] int32: skipped frames ascending in [0, F-A); rest untouched
+ *   d_token_idx  [F*N] int32: f*N + p for each active f (ascending) and p < N,
+ *                in [0, A*N); rest untouched.  May be NULL (not written).
+ *   d_counts     [2] int32: {A, A*N}
+ * Bit-exact; one launch.
+ */
+rf_status rf_schedule_compact(const uint8_t* d_mask, int F, int N, int32_t* d_active,
+                              int32_t* d_skipped, int32_t* d_token_idx, int32_t* d_counts,
+                              rf_stream_t stream);
+
+/*
+ * rf_project -- Eq. 3, latent trajectory projection, for every frame.
+ *
+ *   d_ctx       [F][E] fp32 output: the full-sequence context at sigma_s
+ *   d_z2        [2][F][E] fp32 two-slot store (see conventions)
+ *   d_cur_slot  [F] uint8, 0 or 1
+ *   d_alpha, d_beta  [F] fp32 weights of this step (rf_plan_build row s)
+ *   F, E        frames, elements per frame (E % 4 == 0; 16-byte aligned buffers)
+ * For frame f with cur = z2[cur_slot[f]][f], prev = z2[1-cur_slot[f]][f]:
+ *   beta[f] == 0:  ctx[f] = cur             (active frame: copy, prev not read)
+ *   otherwise:     ctx[f] = fmaf(alpha[f], cur, beta[f]*prev)
+ * d_ctx must not overlap d_z2.
+ */
+rf_status rf_project(float* d_ctx, const float* d_z2, const uint8_t* d_cur_slot,
+                     const float* d_alpha, const float* d_beta, int F, int64_t E,
+                     rf_stream_t stream);
+
+/*
+ * rf_attn -- active-query x full-sequence softmax attention (Sec. 3.2.4 and
+ * Appendix B.2: the active frames' queries attend to the keys and values of
+ * all F*N tokens, true for active frames and projected for skipped ones).
+ *
+ *   d_O          bf16 output, row t at d_O + t*o_row_stride + h*d (t = token);
+ *                only rows of active frames are written
+ *   d_lse        fp32 [H][F*N] natural-log sum-exp per row, or NULL
+ *   d_Q,d_K,d_V  bf16 inputs, row t head h at base + t*qkv_row_stride + h*d
+ *   qkv_row_stride, o_row_stride  elements between tokens (>= H*d, % 8 == 0)
+ *   F, N, H, d   frames, tokens/frame, heads, head dim (d in {64, 128})
+ *   d_active     [F] int32 active frame list, d_counts [2] {A, ...}
+ *                (as written by rf_schedule_compact; read on the device, so no
+ *                host synchronisation is needed between the two calls)
+ *   softmax_scale  scale applied to q.k (e.g. 1/sqrt(d))
+ *   d_status     int32 device word or NULL: set nonzero if a bounded wait in
+ *                the kernel expired (RF_ERR_DEVICE_TIMEOUT in bits 0..7); the
+ *                caller clears it and reads it after synchronising
+ * For each active frame f, token p < N, head h:
+ *   O[f*N+p, h] = sum_j softmax_j(scale * q.k_j) v_j over all F*N tokens j.
+ * Arithmetic: bf16 products, fp32 accumulation and softmax, probabilities
+ * rounded to bf16 for the PV product, output rounded to bf16.
+ * Requires an sm_103 device; bases 16-byte aligned.
+ */
+rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K, const void* d_V,
+                  int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H, int d,
+                  const int32_t* d_active, const int32_t* d_counts, float softmax_scale,
+                  int32_t* d_status, rf_stream_t stream);
+
+/*
+ * rf_step -- heterogeneous flow-matching Euler update (Sec. 3.2.3, Algorithm 2):
+ * each active frame f takes z_next = z + dt[f] * v (dt = sigma_due - sigma_s;
+ * one step for keyframes, n_skip steps for non-keyframes).
+ *
+ *   d_z2        [2][F][E] fp32 two-slot store: reads slot cur_slot[f], writes
+ *               slot 1-cur_slot[f] with fmaf(dt[f], v, z); the caller then flips
+ *               cur_slot[f] for the active frames (rf_plan_build does this)
+ *   d_cur_slot  [F] uint8
+ *   d_v         [F][E] fp32 velocity
+ *   d_dt        [F] fp32
+ *   d_active, d_counts  active list from rf_schedule_compact (device)
+ *   F, E        frames, elements per frame (E % 4 == 0; 16-byte aligned)
+ */
+rf_status rf_step(float* d_z2, const uint8_t* d_cur_slot, const float* d_v, const float* d_dt,
+                  const int32_t* d_active, const int32_t* d_counts, int F, int64_t E,
+                  rf_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RF_H_ */

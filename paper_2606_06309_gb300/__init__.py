@@ -1,0 +1,138 @@
+"""Python binding of librf.so, the RhymeFlow asynchronous step core for GB300.
+
+Argument marshalling only: each function takes torch tensors (or host numpy
+arrays for the planner), passes their raw pointers and sizes to the C ABI
+declared in ``include/rf.h`` and raises ``RFError`` on a non-OK status.  Every
+step of the computation runs in the library's CUDA kernels; there is no CPU or
+PyTorch fallback, and a missing library is an error.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+
+__all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
+           "rf_project", "rf_attn", "rf_step", "rf_status_str", "rf_version", "EXPORTS"]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB: Optional[ctypes.CDLL] = None
+
+# Every symbol include/rf.h declares.
+EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build", "rf_schedule_compact",
+           "rf_project", "rf_attn", "rf_step")
+
+_vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
+_SIG = {
+    "rf_status_str": ([_i32], ctypes.c_char_p),
+    "rf_version": ([], _i32),
+    "rf_last_error": ([], ctypes.c_char_p),
+    "rf_plan_build": ([_i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp], _i32),
+    "rf_schedule_compact": ([_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp], _i32),
+    "rf_project": ([_vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
+    "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
+                 _vp, _vp], _i32),
+    "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
+}
+
+
+class RFError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        detail = load().rf_last_error().decode()
+        super().__init__(f"{fn} failed: {rf_status_str(status)} ({status}): {detail}")
+        self.status = status
+
+
+def lib_path() -> str:
+    return os.path.join(_HERE, "librf.so")
+
+
+def load() -> ctypes.CDLL:
+    """Load librf.so (built by ``build.build()``); raises if it is missing."""
+    global _LIB
+    if _LIB is None:
+        p = lib_path()
+        if not os.path.exists(p):
+            raise RuntimeError(f"{p} is missing: build it with __graft_entry__.build() "
+                               "(there is no fallback implementation)")
+        lib = ctypes.CDLL(p)
+        for name, (args, res) in _SIG.items():
+            f = getattr(lib, name)
+            f.argtypes = args
+            f.restype = res
+        _LIB = lib
+    return _LIB
+
+
+def _check(fn: str, st: int):
+    if st != 0:
+        raise RFError(fn, st)
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def rf_status_str(status: int) -> str:
+    return load().rf_status_str(int(status)).decode()
+
+
+def rf_version() -> int:
+    return load().rf_version()
+
+
+def rf_plan_build(F: int, S: int, is_key, stride, T_w: int, sigma=None):
+    """Host planner.  Returns numpy arrays mask, alpha, beta, dt, cur_slot ([S, F])."""
+    is_key = np.ascontiguousarray(np.asarray(is_key, dtype=np.uint8))
+    stride = np.ascontiguousarray(np.asarray(stride, dtype=np.int32))
+    sig = None if sigma is None else np.ascontiguousarray(np.asarray(sigma, dtype=np.float64))
+    mask = np.zeros((S, F), np.uint8)
+    alpha = np.zeros((S, F), np.float32)
+    beta = np.zeros((S, F), np.float32)
+    dt = np.zeros((S, F), np.float32)
+    slot = np.zeros((S, F), np.uint8)
+    _check("rf_plan_build", load().rf_plan_build(
+        F, S, _ptr(is_key), _ptr(stride), T_w, _ptr(sig), _ptr(mask), _ptr(alpha), _ptr(beta),
+        _ptr(dt), _ptr(slot)))
+    return {"mask": mask, "alpha": alpha, "beta": beta, "dt": dt, "cur_slot": slot}
+
+
+def rf_schedule_compact(mask, F: int, N: int, active, skipped, token_idx, counts, stream=None):
+    _check("rf_schedule_compact", load().rf_schedule_compact(
+        _ptr(mask), F, N, _ptr(active), _ptr(skipped), _ptr(token_idx), _ptr(counts),
+        _stream(stream)))
+
+
+def rf_project(ctx, z2, cur_slot, alpha, beta, F: int, E: int, stream=None):
+    _check("rf_project", load().rf_project(
+        _ptr(ctx), _ptr(z2), _ptr(cur_slot), _ptr(alpha), _ptr(beta), F, E, _stream(stream)))
+
+
+def rf_attn(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: int, H: int,
+            d: int, active, counts, softmax_scale: float, status=None, stream=None):
+    _check("rf_attn", load().rf_attn(
+        _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
+        _ptr(active), _ptr(counts), float(softmax_scale), _ptr(status), _stream(stream)))
+
+
+def rf_step(z2, cur_slot, v, dt, active, counts, F: int, E: int, stream=None):
+    _check("rf_step", load().rf_step(
+        _ptr(z2), _ptr(cur_slot), _ptr(v), _ptr(dt), _ptr(active), _ptr(counts), F, E,
+        _stream(stream)))

@@ -1,0 +1,92 @@
+"""Device state and the four-call sequence of one asynchronous denoising step.
+
+One step s of Algorithm 2 on the device, all on one CUDA stream, no host
+synchronisation:
+
+  1. rf_schedule_compact(mask[s])  -> active / skipped frame lists, token list, counts
+  2. rf_project(...)               -> full-sequence context at sigma_s (Eq. 3)
+  3. rf_attn(...)                  -> active queries x all keys (Q/K/V supplied by the
+                                      caller; the DiT projections that would produce them
+                                      from the context are outside this library)
+  4. rf_step(...)                  -> Euler update of the active frames (two-slot store)
+
+The plan (masks, Eq. 3 weights, step sizes, slot bits) comes from the host
+planner rf_plan_build and is uploaded once.  PyTorch only allocates memory.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import rf_attn, rf_plan_build, rf_project, rf_schedule_compact, rf_step
+
+
+@dataclass
+class Plan:
+    mask: torch.Tensor      # [S, F] uint8
+    alpha: torch.Tensor     # [S, F] fp32
+    beta: torch.Tensor      # [S, F] fp32
+    dt: torch.Tensor        # [S, F] fp32
+    cur_slot: torch.Tensor  # [S, F] uint8
+    host: dict
+
+
+def upload_plan(F, S, is_key, stride, T_w, device, sigma=None) -> Plan:
+    h = rf_plan_build(F, S, is_key, stride, T_w, sigma)
+    t = {k: torch.from_numpy(v).to(device) for k, v in h.items()}
+    return Plan(t["mask"], t["alpha"], t["beta"], t["dt"], t["cur_slot"], h)
+
+
+class StepCore:
+    """Buffers for F frames of N tokens, E latent elements per frame, H heads of dim d."""
+
+    def __init__(self, F: int, N: int, E: int, H: int, d: int, plan: Plan, device="cuda",
+                 token_list: bool = True):
+        self.F, self.N, self.E, self.H, self.d = F, N, E, H, d
+        self.plan = plan
+        dev = torch.device(device)
+        self.active = torch.zeros(F, dtype=torch.int32, device=dev)
+        self.skipped = torch.zeros(F, dtype=torch.int32, device=dev)
+        self.token_idx = torch.zeros(F * N, dtype=torch.int32, device=dev) if token_list else None
+        self.counts = torch.zeros(2, dtype=torch.int32, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.z2 = torch.zeros(2, F, E, dtype=torch.float32, device=dev)
+        self.ctx = torch.zeros(F, E, dtype=torch.float32, device=dev)
+
+    def set_state(self, z0: torch.Tensor):
+        self.z2[0].copy_(z0)
+        self.z2[1].copy_(z0)
+
+    def current(self, s: int) -> torch.Tensor:
+        """State of every frame when step s begins (s = S: the final state)."""
+        S = self.plan.mask.shape[0]
+        if s < S:
+            slot = self.plan.cur_slot[s].long()
+        else:  # after the last step: flip the slots of the frames active at S-1
+            slot = (self.plan.cur_slot[S - 1] ^ self.plan.mask[S - 1]).long()
+        idx = torch.arange(self.F, device=slot.device)
+        return self.z2[slot, idx]
+
+    def compact(self, s: int, stream=None):
+        rf_schedule_compact(self.plan.mask[s], self.F, self.N, self.active, self.skipped,
+                            self.token_idx, self.counts, stream)
+
+    def project(self, s: int, stream=None):
+        rf_project(self.ctx, self.z2, self.plan.cur_slot[s], self.plan.alpha[s],
+                   self.plan.beta[s], self.F, self.E, stream)
+
+    def attn(self, O, Q, K, V, scale: float, lse: Optional[torch.Tensor] = None, stream=None):
+        rf_attn(O, lse, Q, K, V, Q.stride(0), O.stride(0), self.F, self.N, self.H, self.d,
+                self.active, self.counts, scale, self.status, stream)
+
+    def step(self, s: int, v: torch.Tensor, stream=None):
+        rf_step(self.z2, self.plan.cur_slot[s], v, self.plan.dt[s], self.active, self.counts,
+                self.F, self.E, stream)
+
+    def run(self, s: int, v, O, Q, K, V, scale: float, lse=None, stream=None):
+        self.compact(s, stream)
+        self.project(s, stream)
+        self.attn(O, Q, K, V, scale, lse, stream)
+        self.step(s, v, stream)

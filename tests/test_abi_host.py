@@ -1,0 +1,102 @@
+"""CPU tests of the C ABI: the library loads, exports every symbol the header
+declares, the host planner matches the oracle bit for bit, and host-checkable
+argument errors are reported before anything touches a GPU."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "rf.h")
+
+
+@pytest.fixture(scope="module")
+def rf():
+    import paper_2606_06309_gb300 as rf
+    if not os.path.exists(rf.lib_path()):
+        from paper_2606_06309_gb300 import build
+        build.build()
+    rf.load()
+    return rf
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(rf_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(rf):
+    names = _declared()
+    assert set(names) == set(rf.EXPORTS), names
+    lib = ctypes.CDLL(rf.lib_path())
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(rf):
+    assert rf.rf_status_str(0) == "RF_OK"
+    assert rf.rf_status_str(5) == "RF_ERR_DEVICE_TIMEOUT"
+    assert rf.rf_status_str(99) == "RF_ERR_UNKNOWN"
+    assert rf.rf_version() >= 100
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+def test_planner_matches_oracle(rf, name):
+    w = wl.get(name)
+    got = rf.rf_plan_build(w.F, w.S, w.is_key, w.stride, w.T_w)
+    want = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+    np.testing.assert_array_equal(got["mask"], want["mask"])
+    np.testing.assert_array_equal(got["cur_slot"], want["cur_slot"])
+    for k in ("alpha", "beta", "dt"):
+        np.testing.assert_array_equal(got[k], want[k].astype(np.float32), err_msg=k)
+
+
+@pytest.mark.parametrize("T_w", [0, 3, 8])
+def test_planner_warmup_and_sigma(rf, T_w):
+    F, S = 7, 12
+    is_key = [1, 0, 0, 1, 0, 0, 1]
+    stride = wl.progressive_stride(S, 3)
+    sig = np.array([(1 - s / S) ** 1.5 for s in range(S + 1)])  # non-uniform schedule
+    got = rf.rf_plan_build(F, S, is_key, stride, T_w, sig)
+    want = oracle.schedule(F, S, is_key, stride, T_w, sigma=sig)
+    np.testing.assert_array_equal(got["mask"], want["mask"])
+    for k in ("alpha", "beta", "dt"):
+        np.testing.assert_array_equal(got[k], want[k].astype(np.float32), err_msg=k)
+
+
+def test_planner_rejects_bad_args(rf):
+    with pytest.raises(rf.RFError):
+        rf.rf_plan_build(3, 4, [1, 0, 0], [2, 0, 2, 2], 0)       # stride < 1
+    with pytest.raises(rf.RFError):
+        rf.rf_plan_build(3, 4, [1, 0, 0], [2] * 4, 5)            # T_w > S
+    with pytest.raises(rf.RFError):
+        rf.rf_plan_build(3, 2, [1, 0, 0], [2] * 2, 0, [1.0, 0.5, 0.1])  # sigma_S != 0
+
+
+def test_device_calls_reject_bad_args_on_host(rf):
+    """Checks that happen before any CUDA call: null pointers, sizes, head dim."""
+    lib = rf.load()
+    P = 256  # any non-null, 16-byte aligned value; never dereferenced
+    assert lib.rf_schedule_compact(None, 4, 8, P, P, P, P, None) == 1
+    assert lib.rf_schedule_compact(P, 0, 8, P, P, P, P, None) == 1
+    assert lib.rf_project(P, P, P, P, P, 4, 6, None) == 3            # E % 4 != 0
+    assert lib.rf_step(P, P, None, P, P, P, 4, 8, None) == 1
+    args = [P, None, P, P, P, 256, 256, 4, 64, 2, 96, P, P, 0.1, None, None]
+    assert lib.rf_attn(*args) == 2                                   # d = 96 unsupported
+    args[10] = 128
+    args[13] = -1.0
+    assert lib.rf_attn(*args) == 1                                   # scale <= 0
+    args[13] = 0.1
+    args[5] = 100
+    assert lib.rf_attn(*args) == 1                                   # row stride < H*d
+    args[5] = 260
+    assert lib.rf_attn(*args) == 3                                   # row stride % 8 != 0
+    args[5] = 256
+    args[2] = P + 2
+    assert lib.rf_attn(*args) == 3                                   # misaligned Q

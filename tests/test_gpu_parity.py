@@ -1,0 +1,306 @@
+"""GPU parity: every kernel through the C ABI against the fp64 oracle.
+
+Integer outputs (index lists, counts) must match bit for bit; the fp32
+projection and Euler update within 1e-5 relative error measured against the
+magnitude of their terms; bf16 attention within the bounds of attn_check.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as wl
+from attn_check import compare
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+SENTINEL = 7.0  # rows the kernel must not write keep this value
+
+
+def _plan(rf, w):
+    return rf.rf_plan_build(w.F, w.S, w.is_key, w.stride, w.T_w)
+
+
+# ---------------------------------------------------------------------------
+# rf_schedule_compact
+# ---------------------------------------------------------------------------
+def _masks():
+    out = []
+    for name in ("tiny", "small", "mid", "long"):
+        w = wl.get(name)
+        p = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+        for row in np.unique(p["mask"], axis=0):
+            out.append((w.N, row))
+    rng = np.random.default_rng(0)
+    for F in (1, 2, 31, 32, 33, 64, 100, 1000, 4096):
+        out.append((int(rng.integers(1, 200)), (rng.random(F) < 0.4).astype(np.uint8)))
+    out.append((5, np.zeros(9, np.uint8)))
+    out.append((3, np.ones(40, np.uint8)))
+    out.append((1, np.array([1], np.uint8)))
+    return out
+
+
+@pytest.mark.parametrize("case", range(len(_masks())))
+def test_compact_bit_exact(cuda_lib, case):
+    rf = cuda_lib
+    N, mask = _masks()[case]
+    F = len(mask)
+    d_mask = torch.from_numpy(mask).to(DEV)
+    act = torch.full((F,), -1, dtype=torch.int32, device=DEV)
+    skp = torch.full((F,), -1, dtype=torch.int32, device=DEV)
+    tok = torch.full((F * N,), -1, dtype=torch.int32, device=DEV)
+    cnt = torch.full((2,), -1, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(d_mask, F, N, act, skp, tok, cnt)
+    torch.cuda.synchronize()
+    a, s, t, c = oracle.compact(mask, N)
+    A = len(a)
+    assert cnt.cpu().tolist() == c.tolist()
+    assert act.cpu().numpy()[:A].tolist() == a.tolist()
+    assert (act.cpu().numpy()[A:] == -1).all()
+    assert skp.cpu().numpy()[:F - A].tolist() == s.tolist()
+    assert tok.cpu().numpy()[:A * N].tolist() == t.tolist()
+    assert (tok.cpu().numpy()[A * N:] == -1).all()
+
+
+# ---------------------------------------------------------------------------
+# rf_project / rf_step
+# ---------------------------------------------------------------------------
+def _rel_err(g, want, scale):
+    return float((np.abs(g - want) / np.maximum(np.maximum(np.abs(want), scale), 1e-30)).max())
+
+
+@pytest.mark.parametrize("F,E", [(4, 64 * 16), (13, 1560 * 16), (21, 3600 * 16), (3, 4), (5, 1000)])
+def test_project_parity(cuda_lib, F, E):
+    rf = cuda_lib
+    g = torch.Generator().manual_seed(F * 7 + E)
+    z2 = torch.randn(2, F, E, generator=g)
+    slot = (torch.rand(F, generator=g) < 0.5).to(torch.uint8)
+    alpha = torch.rand(F, generator=g)
+    active = torch.rand(F, generator=g) < 0.3
+    alpha[active] = 1.0
+    alpha64 = alpha.double()
+    beta = (1.0 - alpha64).float()
+    ctx = torch.full((F, E), SENTINEL, device=DEV)
+    rf.rf_project(ctx, z2.to(DEV), slot.to(DEV), alpha.to(DEV), beta.to(DEV), F, E)
+    torch.cuda.synchronize()
+    idx = torch.arange(F)
+    cur = z2[slot.long(), idx]
+    prev = z2[1 - slot.long(), idx]
+    want = oracle.project(prev, cur, alpha64.numpy())
+    got = ctx.cpu().double().numpy()
+    terms = np.abs(beta.double().numpy()[:, None] * prev.double().numpy()) + \
+        np.abs(alpha64.numpy()[:, None] * cur.double().numpy())
+    assert _rel_err(got, want, terms) <= 1e-5
+    # active frames are copied exactly
+    np.testing.assert_array_equal(got[active.numpy()], cur.double().numpy()[active.numpy()])
+
+
+@pytest.mark.parametrize("F,E", [(4, 64 * 16), (13, 1560 * 16), (33, 3600 * 16), (2, 4)])
+def test_step_parity(cuda_lib, F, E):
+    rf = cuda_lib
+    g = torch.Generator().manual_seed(F + E)
+    z2 = torch.randn(2, F, E, generator=g)
+    v = torch.randn(F, E, generator=g)
+    slot = (torch.rand(F, generator=g) < 0.5).to(torch.uint8)
+    dt = -torch.rand(F, generator=g)
+    mask = (torch.rand(F, generator=g) < 0.6).to(torch.uint8)
+    mask[0] = 1
+    d_z2 = z2.to(DEV)
+    act = torch.zeros(F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(mask.to(DEV), F, 1, act, skp, None, cnt)
+    rf.rf_step(d_z2, slot.to(DEV), v.to(DEV), dt.to(DEV), act, cnt, F, E)
+    torch.cuda.synchronize()
+    out = d_z2.cpu()
+    idx = torch.arange(F)
+    cur = z2[slot.long(), idx]
+    want = oracle.euler(cur, v, dt.double().numpy())
+    got_new = out[1 - slot.long(), idx].double().numpy()
+    m = mask.numpy().astype(bool)
+    terms = np.abs(cur.double().numpy()) + np.abs(dt.double().numpy()[:, None] * v.double().numpy())
+    assert _rel_err(got_new[m], want[m], terms[m]) <= 1e-5
+    # current slots untouched; inactive frames' other slot untouched
+    np.testing.assert_array_equal(out[slot.long(), idx].numpy(), cur.numpy())
+    np.testing.assert_array_equal(got_new[~m], z2[1 - slot.long(), idx].double().numpy()[~m])
+
+
+# ---------------------------------------------------------------------------
+# rf_attn
+# ---------------------------------------------------------------------------
+def _run_attn(rf, Q, K, V, F, N, mask, scale, O=None, lse=True):
+    H, d = Q.shape[1], Q.shape[2]
+    S_tok = F * N
+    if O is None:
+        O = torch.full((S_tok, H, d), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    L = torch.full((H, S_tok), SENTINEL, dtype=torch.float32, device=DEV) if lse else None
+    act = torch.zeros(F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(torch.as_tensor(np.asarray(mask, np.uint8)).to(DEV), F, N, act, skp,
+                           None, cnt)
+    rf.rf_attn(O, L, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt, scale, status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    return O, L
+
+
+def _active_rows(mask, N):
+    return [f * N + p for f in range(len(mask)) if mask[f] for p in range(N)]
+
+
+def _check_attn(Q, K, V, O, L, mask, N, scale, rows=None, heads=None, label=""):
+    all_rows = _active_rows(mask, N)
+    rows = all_rows if rows is None else rows
+    Oref, Lref = oracle.attention(Q.cpu(), K.cpu(), V.cpu(), rows, scale, heads)
+    hs = slice(None) if heads is None else list(heads)
+    Og = O.cpu().float()[rows][:, hs].numpy()
+    Lg = None if L is None else L.cpu()[hs][:, rows].numpy()
+    stats = compare(Og, Oref, Lg, Lref if L is not None else None, label)
+    # rows of skipped frames are untouched
+    skipped = sorted(set(range(len(mask) * N)) - set(all_rows))
+    if skipped:
+        sk = torch.tensor(skipped[:4096])
+        assert (O.cpu()[sk].float() == SENTINEL).all()
+        if L is not None:
+            assert (L.cpu()[:, sk] == SENTINEL).all()
+    return stats
+
+
+def _qkv(S_tok, H, d, seed, device=DEV):
+    g = torch.Generator(device=device).manual_seed(seed)
+    return [torch.randn(S_tok, H, d, generator=g, device=device).to(torch.bfloat16)
+            for _ in range(3)]
+
+
+def test_attn_tiny_every_step(cuda_lib):
+    rf = cuda_lib
+    w = wl.get("tiny")
+    Q, K, V = (x.to(DEV) for x in wl.qkv(w))
+    p = _plan(rf, w)
+    for s in range(w.S):
+        O, L = _run_attn(rf, Q, K, V, w.F, w.N, p["mask"][s], w.softmax_scale)
+        _check_attn(Q, K, V, O, L, p["mask"][s], w.N, w.softmax_scale, label=f"tiny s={s}")
+
+
+@pytest.mark.parametrize("F,N,H,d,mask", [
+    (3, 1560, 2, 128, [1, 0, 1]),
+    (3, 1560, 2, 128, [0, 1, 0]),
+    (3, 1560, 1, 128, [1, 1, 1]),
+    (5, 100, 2, 64, [1, 0, 1, 1, 0]),     # N % 8 != 0: padded rows
+    (5, 100, 3, 128, [0, 0, 0, 0, 1]),
+    (2, 8, 2, 64, [1, 1]),                # one tile, no second tile
+    (7, 136, 2, 128, [1, 1, 1, 0, 1, 1, 1]),
+    (1, 130, 1, 64, [1]),                 # KV tail of 2 keys
+])
+def test_attn_ragged_shapes(cuda_lib, F, N, H, d, mask):
+    rf = cuda_lib
+    Q, K, V = _qkv(F * N, H, d, seed=F * 1000 + N + d)
+    scale = 1.0 / math.sqrt(d)
+    O, L = _run_attn(rf, Q, K, V, F, N, mask, scale)
+    _check_attn(Q, K, V, O, L, mask, N, scale, label=f"{F}x{N} h{H} d{d} {mask}")
+
+
+def test_attn_no_active_frames(cuda_lib):
+    rf = cuda_lib
+    Q, K, V = _qkv(4 * 64, 2, 64, seed=3)
+    O, L = _run_attn(rf, Q, K, V, 4, 64, [0, 0, 0, 0], 0.125)
+    assert (O.float() == SENTINEL).all() and (L == SENTINEL).all()
+
+
+def test_attn_strided_rows(cuda_lib):
+    """Q, K, V as slices of one fused [tokens, 3, H, d] buffer; O with padded rows."""
+    rf = cuda_lib
+    F, N, H, d = 4, 200, 3, 128
+    g = torch.Generator(device=DEV).manual_seed(11)
+    qkv = torch.randn(F * N, 3, H, d, generator=g, device=DEV).to(torch.bfloat16)
+    Q, K, V = qkv[:, 0], qkv[:, 1], qkv[:, 2]
+    O = torch.full((F * N, H * d + 64), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    Ov = O[:, : H * d].view(F * N, H, d)
+    mask = [1, 0, 0, 1]
+    _run_attn(rf, Q, K, V, F, N, mask, 1 / math.sqrt(d), O=Ov, lse=False)
+    _check_attn(Q, K, V, Ov, None, mask, N, 1 / math.sqrt(d), label="strided")
+    assert (O[:, H * d:].float() == SENTINEL).all()
+
+
+def test_attn_planted_keys(cuda_lib):
+    """q_i = 16 k_{pi(i)}: each output row must be v_{pi(i)} at O(1) scale."""
+    rf = cuda_lib
+    F, N, H, d = 3, 256, 2, 128
+    g = torch.Generator(device=DEV).manual_seed(5)
+    K = torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
+    V = torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
+    perm = torch.randperm(F * N, generator=g, device=DEV)
+    Q = (16.0 * K[perm].float()).to(torch.bfloat16)
+    O, _ = _run_attn(rf, Q, K, V, F, N, [1, 1, 1], 1 / math.sqrt(d))
+    err = (O.float() - V[perm].float()).abs().max().item()
+    assert err < 2e-2, err
+
+
+@pytest.mark.parametrize("name,steps", [("small", (0, 1)), ("large", (0, 1))])
+def test_attn_full_size_sampled_rows(cuda_lib, name, steps):
+    """The benchmark's launch configuration at full size; sampled rows against
+    the oracle: the first and last row of every active frame, the rows around
+    each 128-row tile boundary of the first frame, and seeded random rows."""
+    rf = cuda_lib
+    w = wl.get(name)
+    Q, K, V = wl.qkv(w, device=DEV)
+    p = _plan(rf, w)
+    heads = [0, w.H - 1] if w.H > 2 else list(range(w.H))
+    rng = np.random.default_rng(w.seed)
+    for s in steps:
+        mask = p["mask"][s]
+        O, L = _run_attn(rf, Q, K, V, w.F, w.N, mask, w.softmax_scale)
+        act = [f for f in range(w.F) if mask[f]]
+        rows = set()
+        for f in act:
+            rows.update({f * w.N, f * w.N + w.N - 1})
+        f0 = act[0]
+        for t in range(1, w.N // 128 + 1):
+            rows.update({f0 * w.N + min(t * 128 - 1, w.N - 1), f0 * w.N + min(t * 128, w.N - 1)})
+        all_rows = np.array(_active_rows(mask, w.N))
+        rows.update(rng.choice(all_rows, size=96, replace=False).tolist())
+        rows = sorted(rows)
+        hq = torch.tensor(heads, device=DEV)
+        Qs, Ks, Vs = (x.index_select(1, hq).cpu() for x in (Q, K, V))
+        Oref, Lref = oracle.attention(Qs, Ks, Vs, rows, w.softmax_scale)
+        Og = O.cpu().float()[rows][:, heads].numpy()
+        Lg = L.cpu()[heads][:, rows].numpy()
+        compare(Og, Oref, Lg, Lref, f"{name} s={s}")
+        # every active row written, no skipped row written
+        written = (O[:, heads[0]].float() != SENTINEL).any(dim=1).cpu().numpy()
+        expect = np.zeros(w.S_tok, bool)
+        expect[all_rows] = True
+        assert (written == expect).all()
+
+
+# ---------------------------------------------------------------------------
+# Whole trajectory: compaction + projection + attention + Euler step, S steps
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["tiny", "small"])
+def test_trajectory_matches_oracle_sampler(cuda_lib, name):
+    from paper_2606_06309_gb300.stepcore import StepCore, upload_plan
+    w = wl.get(name)
+    plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, DEV)
+    E = w.N * w.C
+    core = StepCore(w.F, w.N, E, w.H, w.d, plan, DEV)
+    z0 = wl.latents(w)
+    core.set_state(z0.to(DEV))
+    Q, K, V = wl.qkv(w, device=DEV)
+    O = torch.zeros_like(Q)
+    vels = [wl.velocity(w, s) for s in range(w.S)]
+    oplan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+    zT_ref, ctx_ref = oracle.sampler(z0, vels, oplan)
+    for s in range(w.S):
+        core.run(s, vels[s].to(DEV), O, Q, K, V, w.softmax_scale)
+        ctx = core.ctx.cpu().double().numpy()
+        err = np.abs(ctx - ctx_ref[s]).max() / max(np.abs(ctx_ref[s]).max(), 1.0)
+        assert err <= 1e-5, (s, err)
+    got = core.current(w.S).cpu().double().numpy()
+    err = np.abs(got - zT_ref).max() / max(np.abs(zT_ref).max(), 1.0)
+    assert err <= 1e-5, err
+    assert core.status.item() == 0
