@@ -330,9 +330,16 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         for (int c = 0; c < BN; ++c)
           if (c >= valid) sf[c] = -INFINITY;
       }
-      float mx = sf[0];
+      // row max as 8 independent chains (a single 128-long chain is pure latency)
+      float mx8[8];
 #pragma unroll
-      for (int c = 1; c < BN; ++c) mx = fmaxf(mx, sf[c]);
+      for (int i = 0; i < 8; ++i) mx8[i] = sf[i];
+#pragma unroll
+      for (int c = 8; c < BN; c += 8)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], sf[c + i]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float m_new = fmaxf(m, mx * sl2);
       const bool need = m_new > m + kRescaleLog2;
       const bool rescale = __any_sync(0xffffffffu, need);
@@ -343,6 +350,7 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         m = m_new;
       }
       const float nm = -m;
+      float l8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // 8 independent sum chains
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t pk[32];
@@ -350,11 +358,13 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         for (int e = 0; e < 32; ++e) {
           const float p0 = ex2_approx(fmaf(sf[half * 64 + 2 * e], sl2, nm));
           const float p1 = ex2_approx(fmaf(sf[half * 64 + 2 * e + 1], sl2, nm));
-          l += p0 + p1;
+          l8[(2 * e) & 7] += p0;
+          l8[(2 * e + 1) & 7] += p1;
           pk[e] = pack_bf16x2(p0, p1);
         }
         tmem_st32(tS + half * 32, pk);
       }
+      l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
       // O was last written by PV(j-1), which completed before S(j) was signalled
       if (rescale && j > 0) {
 #pragma unroll 1
