@@ -36,10 +36,12 @@ METRIC = "rf_attn TFLOP/s (% BF16 peak); step-core ms vs all-frames-active on 1 
 UNIT = "TFLOP/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM traffic of rf_attn measured with ncu (dram__bytes_read.sum + dram__bytes_write.sum),
-# per launch averaged over one trajectory of the "small" workload, valid only for the kernel
-# source with this hash.
-ATTN_TRAFFIC = {"sha256_rf_attn_cu": None, "workload": "small", "bytes_per_launch": None}
+# DRAM traffic of one rf_attn launch measured with ncu (dram__bytes_read.sum +
+# dram__bytes_write.sum; the capture is summarised in profiles/attn_kernel_small_all_active.md).
+# It is reported only while the kernel source still has this hash.
+ATTN_TRAFFIC = {"sha256_rf_attn_cu": "2fddab2c4fef63dc69189a9fbb89392fed383ece746b3aa010197c040cfcebe0",
+                "workload": "small", "bytes_per_launch": 187561984 + 42736896,
+                "launch": "schedule step 0 of the small workload (all 13 frames active)"}
 
 
 def _env_rank():
@@ -254,6 +256,7 @@ def run_gpu(args):
             "frac": round(achieved / peaks["bf16_tflops"], 4),
             "frac_of_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4),
             "traffic": traffic,
+            "traffic_launch": ATTN_TRAFFIC["launch"] if traffic is not None else None,
             "flops_per_launch": per_launch_flops,
             "avg_launch_ms": round(attn_ms_total / len(ev), 5),
         },

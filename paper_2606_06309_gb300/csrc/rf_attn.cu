@@ -330,14 +330,15 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         for (int c = 0; c < BN; ++c)
           if (c >= valid) sf[c] = -INFINITY;
       }
-      // row max as 8 independent chains (a single 128-long chain is pure latency)
+      // row max: 8 independent chains of three-input maxima (a single 128-long chain of
+      // two-input maxima is pure latency on the path from QK^T to PV)
       float mx8[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = sf[i];
+      for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(sf[i], sf[i + 8]);
 #pragma unroll
-      for (int c = 8; c < BN; c += 8)
+      for (int c = 16; c < BN; c += 16)
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], sf[c + i]);
+        for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], sf[c + i], sf[c + 8 + i]);
       const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                              fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float m_new = fmaxf(m, mx * sl2);
@@ -349,22 +350,30 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         l *= fac;
         m = m_new;
       }
-      const float nm = -m;
-      float l8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // 8 independent sum chains
+      // p = 2^(s*scale*log2(e) - m) with packed fp32 pairs for the scale/subtract and the
+      // row sum (8 independent sum chains in 4 packed accumulators)
+      const uint64_t sl2x2 = f2_pack(sl2, sl2), nmx2 = f2_pack(-m, -m);
+      uint64_t l4[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         uint32_t pk[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
-          const float p0 = ex2_approx(fmaf(sf[half * 64 + 2 * e], sl2, nm));
-          const float p1 = ex2_approx(fmaf(sf[half * 64 + 2 * e + 1], sl2, nm));
-          l8[(2 * e) & 7] += p0;
-          l8[(2 * e + 1) & 7] += p1;
+          float x0, x1;
+          f2_unpack(ffma2(f2_pack(sf[half * 64 + 2 * e], sf[half * 64 + 2 * e + 1]), sl2x2, nmx2),
+                    x0, x1);
+          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          l4[e & 3] = fadd2(l4[e & 3], f2_pack(p0, p1));
           pk[e] = pack_bf16x2(p0, p1);
         }
         tmem_st32(tS + half * 32, pk);
       }
-      l += ((l8[0] + l8[1]) + (l8[2] + l8[3])) + ((l8[4] + l8[5]) + (l8[6] + l8[7]));
+      {
+        const uint64_t t = fadd2(fadd2(l4[0], l4[1]), fadd2(l4[2], l4[3]));
+        float a, b;
+        f2_unpack(t, a, b);
+        l += a + b;
+      }
       // O was last written by PV(j-1), which completed before S(j) was signalled
       if (rescale && j > 0) {
 #pragma unroll 1
