@@ -156,12 +156,29 @@ rf_status rf_project(float* d_ctx, const float* d_z2, const uint8_t* d_cur_slot,
  *   O[f*N+p, h] = sum_j softmax_j(scale * q.k_j) v_j over all F*N tokens j.
  * Arithmetic: bf16 products, fp32 accumulation and softmax, probabilities
  * rounded to bf16 for the PV product, output rounded to bf16.
+ *   d_workspace, workspace_bytes  optional device scratch for split-KV (NULL / 0 =
+ *                no split).  With at least rf_attn_workspace_bytes(d) bytes, 256-byte
+ *                aligned and ZERO-FILLED before its first use, the last, partly
+ *                idle round of work is split into ranges of keys whose partial
+ *                results are merged on the device; the kernel leaves the workspace
+ *                ready for the next call.  Calls that share a workspace must not
+ *                overlap on the GPU (keep them on one stream).  After a call that
+ *                reported RF_ERR_DEVICE_TIMEOUT, zero it again.
  * Requires an sm_103 device; bases 16-byte aligned.
  */
 rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K, const void* d_V,
                   int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H, int d,
                   const int32_t* d_active, const int32_t* d_counts, float softmax_scale,
-                  int32_t* d_status, rf_stream_t stream);
+                  void* d_workspace, int64_t workspace_bytes, int32_t* d_status,
+                  rf_stream_t stream);
+
+/*
+ * rf_attn_workspace_bytes -- bytes of split-KV workspace rf_attn can use on the
+ * current device for head dim d (independent of the problem size: counters plus
+ * one partial result tile per SM).  Returns -1 for an unsupported d or when the
+ * device cannot be queried.
+ */
+int64_t rf_attn_workspace_bytes(int d);
 
 /*
  * rf_step -- heterogeneous flow-matching Euler update (Sec. 3.2.3, Algorithm 2):

@@ -15,14 +15,15 @@ from typing import Optional
 import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_attn", "rf_step", "rf_status_str", "rf_version", "EXPORTS"]
+           "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_step", "rf_status_str",
+           "rf_version", "EXPORTS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB: Optional[ctypes.CDLL] = None
 
 # Every symbol include/rf.h declares.
-EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_attn", "rf_step")
+EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
+           "rf_schedule_compact", "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_step")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
 _SIG = {
@@ -33,7 +34,8 @@ _SIG = {
     "rf_schedule_compact": ([_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp], _i32),
     "rf_project": ([_vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
     "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
-                 _vp, _vp], _i32),
+                 _vp, _i64, _vp, _vp], _i32),
+    "rf_attn_workspace_bytes": ([_i32], _i64),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
 }
 
@@ -126,10 +128,20 @@ def rf_project(ctx, z2, cur_slot, alpha, beta, F: int, E: int, stream=None):
 
 
 def rf_attn(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: int, H: int,
-            d: int, active, counts, softmax_scale: float, status=None, stream=None):
+            d: int, active, counts, softmax_scale: float, workspace=None, status=None,
+            stream=None):
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check("rf_attn", load().rf_attn(
         _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
-        _ptr(active), _ptr(counts), float(softmax_scale), _ptr(status), _stream(stream)))
+        _ptr(active), _ptr(counts), float(softmax_scale), _ptr(workspace), ws_bytes,
+        _ptr(status), _stream(stream)))
+
+
+def rf_attn_workspace_bytes(d: int) -> int:
+    n = load().rf_attn_workspace_bytes(d)
+    if n < 0:
+        raise RFError("rf_attn_workspace_bytes", 1)
+    return n
 
 
 def rf_step(z2, cur_slot, v, dt, active, counts, F: int, E: int, stream=None):

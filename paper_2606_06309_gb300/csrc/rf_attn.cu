@@ -28,7 +28,11 @@
 //
 // Work item = (head, pair of 128-row query tiles) over the flattened list of active rows
 // (each frame padded to a multiple of 8 rows); items are dealt round-robin to the CTAs, so
-// consecutive CTAs share the same head's K/V through L2.
+// consecutive CTAs share the same head's K/V through L2.  When the last round of items would
+// leave more than half of the CTAs idle and the caller supplied a workspace, each item of that
+// round is split into C ranges of KV tiles (split-KV): every range writes its unnormalised
+// O row, running max and sum to the workspace, and the CTA that finishes the last range of an
+// item merges them (counter per item and query tile, reset to zero by the merging CTA).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -44,8 +48,8 @@
 namespace rf {
 namespace {
 
-constexpr int BM = 128;  // query rows per tile
-constexpr int BN = 128;  // keys per KV tile
+constexpr int BM = 128;       // query rows per tile
+constexpr int BN = 128;       // keys per KV tile
 constexpr int kThreads = 384;  // three warpgroups
 // Register split after launch (setmaxnreg): the launch gives 384 x 168 = 64512 registers; the
 // producer/MMA warpgroup drops to 104 and each softmax warpgroup grows to 200:
@@ -56,6 +60,8 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: no legitimate wait comes close
 constexpr uint64_t kDrainLimitNs = 200000000ull;  // 0.2 s for in-flight copies at teardown
 constexpr float kRescaleLog2 = 8.0f;
+constexpr int kMaxSplit = 16;          // KV ranges per split item
+constexpr int kMaxGrid = 1024;         // workspace is sized for at most this many CTAs
 
 template <int D>
 struct Cfg {
@@ -66,13 +72,17 @@ struct Cfg {
   static constexpr int kSlots = (D == 128) ? 4 : 8;
   static constexpr int kOffKV = 2 * kTileBytes;
   static constexpr int kOffBar = kOffKV + kSlots * kTileBytes;
-  // barriers: q_full[2] q_empty[2] kv_full[S] kv_empty[S] s_full[2] p_full[2] o_done[2] drain
+  // barriers: q_full[2] q_empty[2] kv_full[S] kv_empty[S] s_full[2] p_full[2] o_done[2]
+  // group[2] (the 128 threads of one softmax warpgroup) drain
   static constexpr int kBarQFull = 0, kBarQEmpty = 2, kBarKVFull = 4, kBarKVEmpty = 4 + kSlots,
                        kBarSFull = 4 + 2 * kSlots, kBarPFull = kBarSFull + 2,
-                       kBarODone = kBarPFull + 2, kBarDrain = kBarODone + 2,
-                       kNumBars = kBarDrain + 1;
+                       kBarODone = kBarPFull + 2, kBarGroup = kBarODone + 2,
+                       kBarDrain = kBarGroup + 2, kNumBars = kBarDrain + 1;
+  // misc: tmem address, abort flag, merge flags [2 groups][2 alternating slots]
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
-  static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack to align the base
+  static constexpr int kSmemBytes = kOffMisc + 32 + 1024;  // + slack to align the base
+  // split-KV partial row: D unnormalised outputs, running max (log2 units), running sum
+  static constexpr int kPartFloats = D + 4;
 };
 
 struct AttnParams {
@@ -81,24 +91,77 @@ struct AttnParams {
   const int32_t* active;
   const int32_t* counts;
   int32_t* status;
+  int* ws_count;   // [kMaxGrid] merge counters (zero between launches), or null: no split
+  float* ws_part;  // [kMaxGrid][2][BM][D+4] partial rows
   int64_t o_row_stride;
   int F, N, Np, H, S_tok, nkv;
   float scale_log2;
 };
 
-struct Work {
-  int tiles, pairs, items, R;
+// The schedule every role derives identically from the active count on the device.
+struct Sched {
+  int R, tiles, pairs;  // active rows (padded per frame), query tiles and tile pairs per head
+  int T_full;           // items processed whole
+  int C;                // KV ranges per item of the split tail (1: no split)
+  int units;            // T_full + tail items * C
 };
 
-__device__ __forceinline__ Work work_shape(const AttnParams& p) {
+// One unit of work: a tile pair of one head over KV tiles [j0, j1).
+struct Unit {
+  int h, pr, j0, j1;
+  int part;  // split: partial slot (tail item index * C + range), else -1
+  int item;  // split: tail item index
+};
+
+__device__ __forceinline__ Sched make_sched(const AttnParams& p) {
   int A = p.counts[0];
   A = A < 0 ? 0 : (A > p.F ? p.F : A);
-  Work w;
-  w.R = A * p.Np;
-  w.tiles = (w.R + BM - 1) / BM;
-  w.pairs = (w.tiles + 1) / 2;
-  w.items = w.pairs * p.H;
-  return w;
+  Sched s;
+  s.R = A * p.Np;
+  s.tiles = (s.R + BM - 1) / BM;
+  s.pairs = (s.tiles + 1) / 2;
+  const int T = s.pairs * p.H;
+  const int G = gridDim.x;
+  s.T_full = T;
+  s.C = 1;
+  if (T > 0 && p.ws_count != nullptr) {
+    const int rounds = (T + G - 1) / G;
+    const int tail = T - (rounds - 1) * G;
+    int c = G / tail;
+    if (c > kMaxSplit) c = kMaxSplit;
+    if (c > p.nkv) c = p.nkv;
+    if (c >= 2) {
+      s.T_full = (rounds - 1) * G;
+      s.C = c;
+    }
+  }
+  s.units = s.T_full + (T - s.T_full) * s.C;
+  return s;
+}
+
+__device__ __forceinline__ Unit get_unit(const Sched& s, const AttnParams& p, int w) {
+  Unit u;
+  int item;
+  if (w < s.T_full) {
+    item = w;
+    u.j0 = 0;
+    u.j1 = p.nkv;
+    u.part = -1;
+    u.item = -1;
+  } else {
+    const int k = w - s.T_full;
+    const int ti = k / s.C, c = k - ti * s.C;
+    item = s.T_full + ti;
+    // 32-bit arithmetic on purpose (c <= 16, nkv < 2^24): a 64-bit divide here slowed the
+    // single MMA-issuing thread by ~10% even on launches that never split
+    u.j0 = (c * p.nkv) / s.C;
+    u.j1 = ((c + 1) * p.nkv) / s.C;
+    u.part = k;
+    u.item = ti;
+  }
+  u.h = item / s.pairs;
+  u.pr = item - u.h * s.pairs;
+  return u;
 }
 
 __device__ __forceinline__ void flag_error(const AttnParams& p, int where) {
@@ -113,23 +176,32 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
     if (globaltimer_ns() - t0 > kDrainLimitNs) return;
 }
 
+// All 128 threads of one softmax warpgroup meet on an mbarrier (count 128); the wait is
+// bounded like every other wait and its result is warp-uniform.
+__device__ __forceinline__ bool group_sync(uint32_t bar, int& cnt, volatile int* abort) {
+  mbar_arrive(bar);
+  const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, cnt & 1, abort, kWaitLimitNs));
+  ++cnt;
+  return ok;
+}
+
 // ---------------------------------------------------------------------------------------
 // TMA producer (one thread).
 // ---------------------------------------------------------------------------------------
 template <int D>
 __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorMap* tmK,
                                          const CUtensorMap* tmV, const AttnParams& p,
-                                         const Work& wk, uint32_t sQ0, uint32_t sKV0,
+                                         const Sched& sc, uint32_t sQ0, uint32_t sKV0,
                                          uint32_t bar0, volatile int* abort) {
   using C = Cfg<D>;
   auto bar = [&](int i) { return bar0 + 8u * i; };
   int q_cnt[2] = {0, 0};
   int it = 0;
-  for (int w = blockIdx.x; w < wk.items; w += gridDim.x) {
-    const int h = w / wk.pairs, pr = w - h * wk.pairs;
+  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+    const Unit u = get_unit(sc, p, w);
     for (int X = 0; X < 2; ++X) {
-      const int t = 2 * pr + X;
-      if (t >= wk.tiles) break;
+      const int t = 2 * u.pr + X;
+      if (t >= sc.tiles) break;
       if (!mbar_wait(bar(C::kBarQEmpty + X), (q_cnt[X] & 1) ^ 1, abort, kWaitLimitNs)) {
         flag_error(p, 0);
         goto drain;
@@ -140,23 +212,23 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
       for (int b = 0; b < BM / 8; ++b) {
         const int r = t * BM + b * 8;
         int tok = p.S_tok;  // rows past the active list: out of bounds, zero filled
-        if (r < wk.R) {
+        if (r < sc.R) {
           const int a = r / p.Np;
           tok = p.active[a] * p.N + (r - a * p.Np);
         }
 #pragma unroll
         for (int hb = 0; hb < C::kHalves; ++hb)
           tma_load_3d(dst + hb * C::kHalfBytes + b * 1024, tmQ, bar(C::kBarQFull + X), hb * 64,
-                      h, tok);
+                      u.h, tok);
       }
       ++q_cnt[X];
     }
 #pragma unroll 1
-    for (int j = 0; j < p.nkv; ++j) {
+    for (int j = u.j0; j < u.j1; ++j) {
 #pragma unroll
       for (int kv = 0; kv < 2; ++kv) {
-        const int s = it % C::kSlots, u = it / C::kSlots;
-        if (!mbar_wait(bar(C::kBarKVEmpty + s), (u & 1) ^ 1, abort, kWaitLimitNs)) {
+        const int s = it % C::kSlots, n = it / C::kSlots;
+        if (!mbar_wait(bar(C::kBarKVEmpty + s), (n & 1) ^ 1, abort, kWaitLimitNs)) {
           flag_error(p, 1);
           goto drain;
         }
@@ -165,7 +237,7 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
 #pragma unroll
         for (int hb = 0; hb < C::kHalves; ++hb)
           tma_load_3d(dst + hb * C::kHalfBytes, kv ? tmV : tmK, bar(C::kBarKVFull + s), hb * 64,
-                      h, j * BN);
+                      u.h, j * BN);
         ++it;
       }
     }
@@ -202,7 +274,7 @@ __device__ __forceinline__ void mma_pv(uint32_t tO, uint32_t tP, uint32_t sV, ui
 }
 
 template <int D>
-__device__ __forceinline__ void mma_issuer(const AttnParams& p, const Work& wk, uint32_t tmem,
+__device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc, uint32_t tmem,
                                            uint32_t sQ0, uint32_t sKV0, uint32_t bar0,
                                            volatile int* abort) {
   using C = Cfg<D>;
@@ -226,10 +298,10 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Work& wk, 
     tc_fence_after();
     return ok;
   };
-  for (int w = blockIdx.x; w < wk.items; w += gridDim.x) {
-    const int h = w / wk.pairs, pr = w - h * wk.pairs;
-    (void)h;
-    const bool hasB = 2 * pr + 1 < wk.tiles;
+  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+    const Unit u = get_unit(sc, p, w);
+    const bool hasB = 2 * u.pr + 1 < sc.tiles;
+    const int nj = u.j1 - u.j0;
     if (!mbar_wait(bar(C::kBarQFull + 0), q_cnt[0] & 1, abort, kWaitLimitNs)) goto fail;
     ++q_cnt[0];
     if (hasB) {
@@ -250,7 +322,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Work& wk, 
     if (!wait_p(0)) goto fail;
     mma_pv<D>(tO[0], tS[0], sKV0 + sV * C::kTileBytes, 0);
 #pragma unroll 1
-    for (int j = 0; j + 1 < p.nkv; ++j) {
+    for (int j = 0; j + 1 < nj; ++j) {
       if (!next_slot(sK)) goto fail;
       mma_qk<D>(tS[0], sQ[0], sKV0 + sK * C::kTileBytes);
       tc_commit(bar(C::kBarSFull + 0));
@@ -272,7 +344,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Work& wk, 
     tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       if (!wait_p(1)) goto fail;
-      mma_pv<D>(tO[1], tS[1], sKV0 + sV * C::kTileBytes, p.nkv > 1);
+      mma_pv<D>(tO[1], tS[1], sKV0 + sV * C::kTileBytes, nj > 1);
       tc_commit(bar(C::kBarODone + 1));
       tc_commit(bar(C::kBarQEmpty + 1));
     }
@@ -291,9 +363,23 @@ drain:
 // Softmax / epilogue warpgroup (128 threads, thread = query row of tile X).
 // ---------------------------------------------------------------------------------------
 template <int D>
-__device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& wk, int X,
-                                              uint32_t tmem, uint32_t bar0,
-                                              volatile int* abort) {
+__device__ __forceinline__ void store_row_bf16(uint16_t* orow, const float* o, float scale) {
+  uint4* dst = reinterpret_cast<uint4*>(orow);
+#pragma unroll
+  for (int q = 0; q < D / 8; ++q) {
+    uint4 v;
+    v.x = pack_bf16x2(o[8 * q + 0] * scale, o[8 * q + 1] * scale);
+    v.y = pack_bf16x2(o[8 * q + 2] * scale, o[8 * q + 3] * scale);
+    v.z = pack_bf16x2(o[8 * q + 4] * scale, o[8 * q + 5] * scale);
+    v.w = pack_bf16x2(o[8 * q + 6] * scale, o[8 * q + 7] * scale);
+    dst[q] = v;
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& sc, int X,
+                                              uint32_t tmem, uint32_t bar0, volatile int* abort,
+                                              volatile int* merge_flag) {
   using C = Cfg<D>;
   auto bar = [&](int i) { return bar0 + 8u * i; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -303,14 +389,14 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
   const uint32_t tS = tmem + lane_base + X * 128;
   const uint32_t tO = tmem + lane_base + 256 + X * 128;
   const float sl2 = p.scale_log2;
-  int s_cnt = 0, o_cnt = 0;
-  for (int w = blockIdx.x; w < wk.items; w += gridDim.x) {
-    const int h = w / wk.pairs, pr = w - h * wk.pairs;
-    const int t = 2 * pr + X;
-    if (t >= wk.tiles) continue;
+  int s_cnt = 0, o_cnt = 0, g_cnt = 0, split_cnt = 0;
+  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+    const Unit u = get_unit(sc, p, w);
+    const int t = 2 * u.pr + X;
+    if (t >= sc.tiles) continue;
     float m = -INFINITY, l = 0.f;
 #pragma unroll 1
-    for (int j = 0; j < p.nkv; ++j) {
+    for (int j = u.j0; j < u.j1; ++j) {
       // the result is made warp-uniform: tcgen05.ld/st below are warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(bar(C::kBarSFull + X), s_cnt & 1, abort,
                                             kWaitLimitNs))) {
@@ -369,13 +455,13 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
         tmem_st32(tS + half * 32, pk);
       }
       {
-        const uint64_t t = fadd2(fadd2(l4[0], l4[1]), fadd2(l4[2], l4[3]));
+        const uint64_t t2 = fadd2(fadd2(l4[0], l4[1]), fadd2(l4[2], l4[3]));
         float a, b;
-        f2_unpack(t, a, b);
+        f2_unpack(t2, a, b);
         l += a + b;
       }
       // O was last written by PV(j-1), which completed before S(j) was signalled
-      if (rescale && j > 0) {
+      if (rescale && j > u.j0) {
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           uint32_t o[32];
@@ -390,7 +476,7 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
       tc_fence_before();
       mbar_arrive(bar(C::kBarPFull + X));
     }
-    // epilogue: O / l -> bf16
+    // epilogue
     if (!__all_sync(0xffffffffu,
                     mbar_wait(bar(C::kBarODone + X), o_cnt & 1, abort, kWaitLimitNs))) {
       flag_error(p, 4);
@@ -399,35 +485,96 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Work& w
     ++o_cnt;
     tc_fence_after();
     const int r = t * BM + row;
-    bool valid = r < wk.R;
+    bool valid = r < sc.R;
     int64_t token = 0;
     if (valid) {
       const int a = r / p.Np, pp = r - a * p.Np;
       valid = pp < p.N;
       token = static_cast<int64_t>(p.active[a]) * p.N + pp;
     }
-    const float inv_l = 1.0f / l;
-    uint16_t* orow = p.O + token * p.o_row_stride + static_cast<int64_t>(h) * D;
+    uint16_t* orow = p.O + token * p.o_row_stride + static_cast<int64_t>(u.h) * D;
+    if (u.part < 0) {
+      // whole item: O / l -> bf16
+      const float inv_l = 1.0f / l;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tO + c * 32, o);
+        tmem_wait_ld();
+        if (valid) store_row_bf16<32>(orow + c * 32, reinterpret_cast<const float*>(o), inv_l);
+      }
+      if (valid && p.lse)
+        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] = (m + __log2f(l)) * 0.69314718055994531f;
+      continue;
+    }
+    // split item: publish this KV range's partial row, then the last range to finish merges
+    float* part = p.ws_part + ((static_cast<int64_t>(u.part) * 2 + X) * BM + row) * C::kPartFloats;
 #pragma unroll 1
     for (int c = 0; c < D / 32; ++c) {
       uint32_t o[32];
       tmem_ld32(tO + c * 32, o);
       tmem_wait_ld();
-      if (valid) {
-        uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+      float4* dst = reinterpret_cast<float4*>(part + c * 32);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint4 v;
-          v.x = pack_bf16x2(__uint_as_float(o[8 * q + 0]) * inv_l, __uint_as_float(o[8 * q + 1]) * inv_l);
-          v.y = pack_bf16x2(__uint_as_float(o[8 * q + 2]) * inv_l, __uint_as_float(o[8 * q + 3]) * inv_l);
-          v.z = pack_bf16x2(__uint_as_float(o[8 * q + 4]) * inv_l, __uint_as_float(o[8 * q + 5]) * inv_l);
-          v.w = pack_bf16x2(__uint_as_float(o[8 * q + 6]) * inv_l, __uint_as_float(o[8 * q + 7]) * inv_l);
-          dst[q] = v;
-        }
-      }
+      for (int q = 0; q < 8; ++q)
+        __stcg(dst + q, make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
+                                    __uint_as_float(o[4 * q + 2]), __uint_as_float(o[4 * q + 3])));
     }
-    if (valid && p.lse)
-      p.lse[static_cast<int64_t>(h) * p.S_tok + token] = (m + __log2f(l)) * 0.69314718055994531f;
+    __stcg(reinterpret_cast<float4*>(part + D), make_float4(m, l, 0.f, 0.f));
+    __threadfence();
+    // two flag slots alternate, so a slot is rewritten only after every thread read it
+    volatile int* flag = merge_flag + (split_cnt & 1);
+    ++split_cnt;
+    if (!group_sync(bar(C::kBarGroup + X), g_cnt, abort)) {  // every row is published
+      flag_error(p, 5);
+      return;
+    }
+    if (row == 0) {
+      const int old = atomicAdd(p.ws_count + 2 * u.item + X, 1);
+      *flag = (old == sc.C - 1);
+    }
+    if (!group_sync(bar(C::kBarGroup + X), g_cnt, abort)) {  // the flag is visible
+      flag_error(p, 6);
+      return;
+    }
+    if (*flag == 0) continue;
+    __threadfence();
+    if (valid) {
+      const float* base =
+          p.ws_part + ((static_cast<int64_t>(u.item) * sc.C * 2 + X) * BM + row) * C::kPartFloats;
+      const int64_t stride = static_cast<int64_t>(2) * BM * C::kPartFloats;  // next range
+      // O = sum_c 2^(m_c - M) O_c / sum_c 2^(m_c - M) l_c, M = max_c m_c
+      float M = -INFINITY;
+      for (int c = 0; c < sc.C; ++c) M = fmaxf(M, __ldcg(base + c * stride + D));
+      float L = 0.f;
+      for (int c = 0; c < sc.C; ++c) {
+        const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + c * stride + D));
+        L += ml.y * ex2_approx(ml.x - M);
+      }
+      const float inv_L = 1.0f / L;
+#pragma unroll 1
+      for (int cc = 0; cc < D / 32; ++cc) {
+        float acc[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) acc[e] = 0.f;
+        for (int c = 0; c < sc.C; ++c) {
+          const float* pc = base + c * stride;
+          const float wgt = ex2_approx(__ldcg(pc + D) - M);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 v = __ldcg(reinterpret_cast<const float4*>(pc + cc * 32) + q);
+            acc[4 * q] = fmaf(v.x, wgt, acc[4 * q]);
+            acc[4 * q + 1] = fmaf(v.y, wgt, acc[4 * q + 1]);
+            acc[4 * q + 2] = fmaf(v.z, wgt, acc[4 * q + 2]);
+            acc[4 * q + 3] = fmaf(v.w, wgt, acc[4 * q + 3]);
+          }
+        }
+        store_row_bf16<32>(orow + cc * 32, acc, inv_L);
+      }
+      if (p.lse)
+        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] = (M + __log2f(L)) * 0.69314718055994531f;
+    }
+    if (row == 0) p.ws_count[2 * u.item + X] = 0;  // ready for the next launch
   }
 }
 
@@ -444,6 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sQ0 = sbase, sKV0 = sbase + C::kOffKV, bar0 = sbase + C::kOffBar;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+  volatile int* merge_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 8);  // [2][2]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -453,6 +601,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar0 + 8 * (C::kBarSFull + X), 1);
       mbar_init(bar0 + 8 * (C::kBarPFull + X), 128);
       mbar_init(bar0 + 8 * (C::kBarODone + X), 1);
+      mbar_init(bar0 + 8 * (C::kBarGroup + X), 128);
+      merge_flag[2 * X] = 0;
+      merge_flag[2 * X + 1] = 0;
     }
     for (int s = 0; s < C::kSlots; ++s) {
       mbar_init(bar0 + 8 * (C::kBarKVFull + s), 1);
@@ -473,22 +624,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const Work wk = work_shape(p);
+  const Sched sc = make_sched(p);
 
   // Every warp of warpgroup 0 gives registers back before any softmax warp asks for more,
   // so the increase below always finds them.
   if (warp < 4) {
     reg_dealloc<kRegsControl>();
     if (warp == 0) {
-      if (lane == 0) producer<D>(&tmQ, &tmK, &tmV, p, wk, sQ0, sKV0, bar0, abort);
+      if (lane == 0) producer<D>(&tmQ, &tmK, &tmV, p, sc, sQ0, sKV0, bar0, abort);
       __syncwarp();
     } else if (warp == 1) {
-      if (lane == 0) mma_issuer<D>(p, wk, tmem, sQ0, sKV0, bar0, abort);
+      if (lane == 0) mma_issuer<D>(p, sc, tmem, sQ0, sKV0, bar0, abort);
       __syncwarp();
     }
   } else {
     reg_alloc<kRegsSoftmax>();
-    softmax_group<D>(p, wk, (warp - 4) >> 2, tmem, bar0, abort);
+    const int X = (warp - 4) >> 2;
+    softmax_group<D>(p, sc, X, tmem, bar0, abort, merge_flag + 2 * X);
   }
 
   tc_fence_before();
@@ -538,9 +690,15 @@ rf_status make_map(CUtensorMap* m, const void* base, int d, int H, int S_tok, in
   return RF_OK;
 }
 
+// Workspace layout: [kMaxGrid] int merge counters, then (256-byte aligned) the partial rows.
+constexpr int64_t kCountBytes = kMaxGrid * 4;
+int64_t workspace_bytes(int d, int grid) {
+  return kCountBytes + static_cast<int64_t>(grid) * 2 * BM * (d + 4) * 4;
+}
+
 template <int D>
 rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
-                 const AttnParams& p, const DeviceInfo& di, cudaStream_t stream) {
+                 const AttnParams& p, int grid, const DeviceInfo& di, cudaStream_t stream) {
   using C = Cfg<D>;
   static bool attr_set[64] = {};
   if (C::kSmemBytes > di.max_smem_optin) return fail(RF_ERR_UNSUPPORTED, "shared memory");
@@ -550,12 +708,6 @@ rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& 
       return fail(RF_ERR_CUDA, "cudaFuncSetAttribute(attn_kernel)", e);
     attr_set[di.device] = true;
   }
-  const int64_t rows = static_cast<int64_t>(p.F) * p.Np;
-  const int64_t tiles = (rows + BM - 1) / BM;
-  const int64_t max_items = ((tiles + 1) / 2) * p.H;
-  int grid = di.sm_count;
-  if (max_items < grid) grid = static_cast<int>(max_items);
-  if (grid < 1) grid = 1;
   attn_kernel<D><<<grid, kThreads, C::kSmemBytes, stream>>>(q, k, v, p);
   return launch_status("attn_kernel launch");
 }
@@ -565,10 +717,19 @@ rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& 
 
 using namespace rf;
 
+extern "C" int64_t rf_attn_workspace_bytes(int d) {
+  if (d != 64 && d != 128) return -1;
+  DeviceInfo di;
+  if (current_device_info(&di) != RF_OK) return -1;
+  const int grid = di.sm_count < kMaxGrid ? di.sm_count : kMaxGrid;
+  return workspace_bytes(d, grid);
+}
+
 extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
                              const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride, int F,
                              int N, int H, int d, const int32_t* d_active,
-                             const int32_t* d_counts, float softmax_scale, int32_t* d_status,
+                             const int32_t* d_counts, float softmax_scale, void* d_workspace,
+                             int64_t workspace_bytes_given, int32_t* d_status,
                              rf_stream_t stream) {
   if (!d_O || !d_Q || !d_K || !d_V || !d_active || !d_counts) return RF_ERR_INVALID_ARG;
   if (F < 1 || N < 1 || H < 1 || H > 65535) return RF_ERR_INVALID_ARG;
@@ -583,6 +744,10 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   if (qkv_row_stride % 8 != 0 || o_row_stride % 8 != 0) return RF_ERR_MISALIGNED;
   if (!aligned16(d_Q) || !aligned16(d_K) || !aligned16(d_V) || !aligned16(d_O))
     return RF_ERR_MISALIGNED;
+  if (d_workspace) {
+    if (workspace_bytes_given < 0) return RF_ERR_INVALID_ARG;
+    if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return RF_ERR_MISALIGNED;
+  }
   DeviceInfo di;
   if (rf_status st = current_device_info(&di)) return st;
   if (di.cc_major != 10 || di.cc_minor != 3) return fail(RF_ERR_UNSUPPORTED, "needs sm_103");
@@ -592,12 +757,25 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   if (rf_status st = make_map(&mk, d_K, d, H, static_cast<int>(S_tok), qkv_row_stride, BN)) return st;
   if (rf_status st = make_map(&mv, d_V, d, H, static_cast<int>(S_tok), qkv_row_stride, BN)) return st;
 
+  // Persistent grid: one CTA per SM, fewer if the largest possible active set has fewer items.
+  const int64_t rows = static_cast<int64_t>(F) * Np;
+  const int64_t tiles = (rows + BM - 1) / BM;
+  const int64_t max_items = ((tiles + 1) / 2) * H;
+  int grid = di.sm_count < kMaxGrid ? di.sm_count : kMaxGrid;
+  const bool split = d_workspace != nullptr && workspace_bytes_given >= workspace_bytes(d, grid);
+  // without split-KV there is no use for more CTAs than items
+  if (!split && max_items < grid) grid = static_cast<int>(max_items);
+  if (grid < 1) grid = 1;
+
   AttnParams p;
   p.O = static_cast<uint16_t*>(d_O);
   p.lse = d_lse;
   p.active = d_active;
   p.counts = d_counts;
   p.status = d_status;
+  p.ws_count = split ? static_cast<int*>(d_workspace) : nullptr;
+  p.ws_part = split ? reinterpret_cast<float*>(static_cast<char*>(d_workspace) + kCountBytes)
+                    : nullptr;
   p.o_row_stride = o_row_stride;
   p.F = F;
   p.N = N;
@@ -607,5 +785,5 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   p.nkv = static_cast<int>((S_tok + BN - 1) / BN);
   p.scale_log2 = static_cast<float>(static_cast<double>(softmax_scale) * 1.4426950408889634);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  return d == 128 ? launch<128>(mq, mk, mv, p, di, s) : launch<64>(mq, mk, mv, p, di, s);
+  return d == 128 ? launch<128>(mq, mk, mv, p, grid, di, s) : launch<64>(mq, mk, mv, p, grid, di, s);
 }

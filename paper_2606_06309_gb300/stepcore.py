@@ -20,7 +20,8 @@ from typing import Optional
 
 import torch
 
-from . import rf_attn, rf_plan_build, rf_project, rf_schedule_compact, rf_step
+from . import (rf_attn, rf_attn_workspace_bytes, rf_plan_build, rf_project, rf_schedule_compact,
+               rf_step)
 
 
 @dataclass
@@ -43,7 +44,7 @@ class StepCore:
     """Buffers for F frames of N tokens, E latent elements per frame, H heads of dim d."""
 
     def __init__(self, F: int, N: int, E: int, H: int, d: int, plan: Plan, device="cuda",
-                 token_list: bool = True):
+                 token_list: bool = True, split_kv: bool = True):
         self.F, self.N, self.E, self.H, self.d = F, N, E, H, d
         self.plan = plan
         dev = torch.device(device)
@@ -54,6 +55,11 @@ class StepCore:
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.z2 = torch.zeros(2, F, E, dtype=torch.float32, device=dev)
         self.ctx = torch.zeros(F, E, dtype=torch.float32, device=dev)
+        # split-KV workspace for rf_attn: zero-filled once, left zeroed by every call
+        self.workspace = None
+        if split_kv:
+            nbytes = rf_attn_workspace_bytes(d)
+            self.workspace = torch.zeros((nbytes + 3) // 4, dtype=torch.int32, device=dev)
 
     def set_state(self, z0: torch.Tensor):
         self.z2[0].copy_(z0)
@@ -79,7 +85,7 @@ class StepCore:
 
     def attn(self, O, Q, K, V, scale: float, lse: Optional[torch.Tensor] = None, stream=None):
         rf_attn(O, lse, Q, K, V, Q.stride(0), O.stride(0), self.F, self.N, self.H, self.d,
-                self.active, self.counts, scale, self.status, stream)
+                self.active, self.counts, scale, self.workspace, self.status, stream)
 
     def step(self, s: int, v: torch.Tensor, stream=None):
         rf_step(self.z2, self.plan.cur_slot[s], v, self.plan.dt[s], self.active, self.counts,

@@ -87,7 +87,7 @@ def test_device_calls_reject_bad_args_on_host(rf):
     assert lib.rf_schedule_compact(P, 0, 8, P, P, P, P, None) == 1
     assert lib.rf_project(P, P, P, P, P, 4, 6, None) == 3            # E % 4 != 0
     assert lib.rf_step(P, P, None, P, P, P, 4, 8, None) == 1
-    args = [P, None, P, P, P, 256, 256, 4, 64, 2, 96, P, P, 0.1, None, None]
+    args = [P, None, P, P, P, 256, 256, 4, 64, 2, 96, P, P, 0.1, None, 0, None, None]
     assert lib.rf_attn(*args) == 2                                   # d = 96 unsupported
     args[10] = 128
     args[13] = -1.0
@@ -100,3 +100,9 @@ def test_device_calls_reject_bad_args_on_host(rf):
     args[5] = 256
     args[2] = P + 2
     assert lib.rf_attn(*args) == 3                                   # misaligned Q
+    args[2] = P
+    args[14], args[15] = P + 16, 1 << 30
+    assert lib.rf_attn(*args) == 3                                   # workspace not 256-aligned
+    args[14], args[15] = P, -1
+    assert lib.rf_attn(*args) == 1                                   # negative workspace size
+    assert lib.rf_attn_workspace_bytes(96) == -1

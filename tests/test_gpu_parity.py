@@ -131,7 +131,18 @@ def test_step_parity(cuda_lib, F, E):
 # ---------------------------------------------------------------------------
 # rf_attn
 # ---------------------------------------------------------------------------
-def _run_attn(rf, Q, K, V, F, N, mask, scale, O=None, lse=True):
+_WS = {}
+
+
+def _workspace(rf, d):
+    """Split-KV workspace, zero-filled once per head dim and reused by every call."""
+    if d not in _WS:
+        n = rf.rf_attn_workspace_bytes(d)
+        _WS[d] = torch.zeros((n + 3) // 4, dtype=torch.int32, device=DEV)
+    return _WS[d]
+
+
+def _run_attn(rf, Q, K, V, F, N, mask, scale, O=None, lse=True, split=True):
     H, d = Q.shape[1], Q.shape[2]
     S_tok = F * N
     if O is None:
@@ -143,9 +154,12 @@ def _run_attn(rf, Q, K, V, F, N, mask, scale, O=None, lse=True):
     status = torch.zeros(1, dtype=torch.int32, device=DEV)
     rf.rf_schedule_compact(torch.as_tensor(np.asarray(mask, np.uint8)).to(DEV), F, N, act, skp,
                            None, cnt)
-    rf.rf_attn(O, L, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt, scale, status)
+    ws = _workspace(rf, d) if split else None
+    rf.rf_attn(O, L, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt, scale, ws, status)
     torch.cuda.synchronize()
     assert status.item() == 0
+    if ws is not None:
+        assert int(ws[:1024].abs().sum()) == 0, "merge counters not reset"
     return O, L
 
 
@@ -304,3 +318,30 @@ def test_trajectory_matches_oracle_sampler(cuda_lib, name):
     err = np.abs(got - zT_ref).max() / max(np.abs(zT_ref).max(), 1.0)
     assert err <= 1e-5, err
     assert core.status.item() == 0
+
+
+@pytest.mark.parametrize("F,N,H,d,mask", [
+    (3, 1560, 2, 128, [1, 0, 1]),
+    (5, 100, 2, 64, [1, 0, 1, 1, 0]),
+    (13, 1560, 12, 128, [1] * 13),        # 960 items: the last round is split 3 ways
+])
+def test_attn_split_and_unsplit_agree_with_oracle(cuda_lib, F, N, H, d, mask):
+    """The same call with and without the split-KV workspace: both within tolerance of the
+    oracle (sampled rows for the large case), and close to each other."""
+    rf = cuda_lib
+    Q, K, V = _qkv(F * N, H, d, seed=F + N + d)
+    scale = 1.0 / math.sqrt(d)
+    O1, L1 = _run_attn(rf, Q, K, V, F, N, mask, scale, split=True)
+    O2, L2 = _run_attn(rf, Q, K, V, F, N, mask, scale, split=False)
+    rows = _active_rows(mask, N)
+    if len(rows) > 2048:
+        rng = np.random.default_rng(0)
+        rows = sorted(rng.choice(rows, 256, replace=False).tolist() + [rows[-1], rows[0]])
+    heads = list(range(min(H, 2)))
+    hq = torch.tensor(heads, device=DEV)
+    Qs, Ks, Vs = (x.index_select(1, hq).cpu() for x in (Q, K, V))
+    Oref, Lref = oracle.attention(Qs, Ks, Vs, rows, scale)
+    for O, L, lab in ((O1, L1, "split"), (O2, L2, "unsplit")):
+        compare(O.cpu().float()[rows][:, heads].numpy(), Oref, L.cpu()[heads][:, rows].numpy(),
+                Lref, lab)
+    assert (O1.float() - O2.float()).abs().max().item() < 1e-2
