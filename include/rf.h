@@ -181,6 +181,37 @@ rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K, con
 int64_t rf_attn_workspace_bytes(int d);
 
 /*
+ * rf_attn_noalloc -- rf_attn for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart to this entry point; it exists for deployment.
+ * Some callers of this library cannot call cudaMalloc: code running inside
+ * another engine's execution callback that forbids allocation, serving loops
+ * that must not take cudaMalloc's implicit device-wide synchronisation, or plain
+ * C hosts with no device allocator of their own.  For them this call takes the
+ * same arguments as rf_attn minus the workspace, and uses instead a scratch
+ * array that the library itself holds in device memory: a file-scope array of
+ * 21,630,976 bytes (split-KV counters plus partial tiles for head dim <= 128 on
+ * up to 160 SMs), present on every GPU that loads the library until the
+ * process exits.  The call allocates and frees nothing.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current and caches it; make that
+ *     first call before any stream capture.
+ *   - Each call zeroes the array's counters on `stream` before the kernel runs.
+ *   - Every call on a device shares the one array, and it keeps the last call's
+ *     contents: calls that overlap on the GPU (different streams, or several
+ *     host threads) race on it and give wrong results.  Issue them in order on
+ *     one stream.
+ *   - If the device needs more scratch than the array holds (more than 160
+ *     SMs), the call returns RF_ERR_UNSUPPORTED with the sizes in
+ *     rf_last_error(); nothing is enqueued.
+ * The inputs, outputs and results are those of rf_attn with a workspace.
+ */
+rf_status rf_attn_noalloc(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
+                          const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride, int F,
+                          int N, int H, int d, const int32_t* d_active, const int32_t* d_counts,
+                          float softmax_scale, int32_t* d_status, rf_stream_t stream);
+
+/*
  * rf_step -- heterogeneous flow-matching Euler update (Sec. 3.2.3, Algorithm 2):
  * each active frame f takes z_next = z + dt[f] * v (dt = sigma_due - sigma_s;
  * one step for keyframes, n_skip steps for non-keyframes).

@@ -15,7 +15,8 @@ from typing import Optional
 import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_step", "rf_status_str",
+           "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
+           "rf_status_str",
            "rf_version", "EXPORTS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -23,7 +24,8 @@ _LIB: Optional[ctypes.CDLL] = None
 
 # Every symbol include/rf.h declares.
 EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
-           "rf_schedule_compact", "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_step")
+           "rf_schedule_compact", "rf_project", "rf_attn", "rf_attn_workspace_bytes",
+           "rf_attn_noalloc", "rf_step")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
 _SIG = {
@@ -36,6 +38,8 @@ _SIG = {
     "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
                  _vp, _i64, _vp, _vp], _i32),
     "rf_attn_workspace_bytes": ([_i32], _i64),
+    "rf_attn_noalloc": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
+                         _f32, _vp, _vp], _i32),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
 }
 
@@ -135,6 +139,15 @@ def rf_attn(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: 
         _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
         _ptr(active), _ptr(counts), float(softmax_scale), _ptr(workspace), ws_bytes,
         _ptr(status), _stream(stream)))
+
+
+def rf_attn_noalloc(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: int,
+                    H: int, d: int, active, counts, softmax_scale: float, status=None,
+                    stream=None):
+    """rf_attn for callers that cannot allocate: the library's own static scratch."""
+    _check("rf_attn_noalloc", load().rf_attn_noalloc(
+        _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
+        _ptr(active), _ptr(counts), float(softmax_scale), _ptr(status), _stream(stream)))
 
 
 def rf_attn_workspace_bytes(d: int) -> int:

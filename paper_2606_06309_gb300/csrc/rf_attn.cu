@@ -712,6 +712,16 @@ rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& 
   return launch_status("attn_kernel launch");
 }
 
+// Scratch for rf_attn_noalloc: a file-scope device array, so that callers who cannot allocate
+// device memory still get split-KV.  Sized for head dim 128 on up to 160 SMs (20.6 MiB); every
+// GPU that loads this library holds it until the process exits.
+constexpr int kNoAllocMaxGrid = 160;
+constexpr int64_t kNoAllocScratchBytes =
+    kCountBytes + static_cast<int64_t>(kNoAllocMaxGrid) * 2 * BM * (128 + 4) * 4;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[64] = {};  // device address of the array, per device ordinal
+
 }  // namespace
 }  // namespace rf
 
@@ -786,4 +796,43 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   p.scale_log2 = static_cast<float>(static_cast<double>(softmax_scale) * 1.4426950408889634);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return d == 128 ? launch<128>(mq, mk, mv, p, grid, di, s) : launch<64>(mq, mk, mv, p, grid, di, s);
+}
+
+// rf_attn without any device allocation: the split-KV scratch is the library's own static
+// array.  Host code cannot pass the array's name to a kernel (in host code it only stands in
+// for the symbol), so its device address is looked up once per device and cached.
+extern "C" rf_status rf_attn_noalloc(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
+                                     const void* d_V, int64_t qkv_row_stride,
+                                     int64_t o_row_stride, int F, int N, int H, int d,
+                                     const int32_t* d_active, const int32_t* d_counts,
+                                     float softmax_scale, int32_t* d_status, rf_stream_t stream) {
+  int dev = 0;
+  if (cudaError_t e = cudaGetDevice(&dev)) return fail(RF_ERR_CUDA, "cudaGetDevice", e);
+  if (dev < 0 || dev >= 64) return fail(RF_ERR_UNSUPPORTED, "device ordinal >= 64");
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+      void* ptr = nullptr;
+      if (cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch))
+        return fail(RF_ERR_CUDA, "cudaGetSymbolAddress(rf_attn_noalloc scratch)", e);
+      g_noalloc_addr[dev] = ptr;
+    }
+    scratch = g_noalloc_addr[dev];
+  }
+  const int64_t need = rf_attn_workspace_bytes(d);
+  if (need < 0) return d != 64 && d != 128 ? RF_ERR_UNSUPPORTED : RF_ERR_CUDA;
+  if (need > kNoAllocScratchBytes) {
+    char buf[160];
+    std::snprintf(buf, sizeof(buf),
+                  "rf_attn_noalloc: this device needs %lld bytes of split-KV scratch, the static "
+                  "maximum is %lld",
+                  static_cast<long long>(need), static_cast<long long>(kNoAllocScratchBytes));
+    return fail(RF_ERR_UNSUPPORTED, buf);
+  }
+  // The array keeps whatever the previous call left; the merge counters must start at zero.
+  if (cudaError_t e = cudaMemsetAsync(scratch, 0, kCountBytes, reinterpret_cast<cudaStream_t>(stream)))
+    return fail(RF_ERR_CUDA, "cudaMemsetAsync(rf_attn_noalloc counters)", e);
+  return rf_attn(d_O, d_lse, d_Q, d_K, d_V, qkv_row_stride, o_row_stride, F, N, H, d, d_active,
+                 d_counts, softmax_scale, scratch, kNoAllocScratchBytes, d_status, stream);
 }
