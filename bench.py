@@ -39,8 +39,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic of one rf_attn launch measured with ncu (dram__bytes_read.sum +
 # dram__bytes_write.sum; the capture is summarised in profiles/attn_kernel_small_all_active.md).
 # It is reported only while the kernel source still has this hash.
-ATTN_TRAFFIC = {"sha256_rf_attn_cu": "2fddab2c4fef63dc69189a9fbb89392fed383ece746b3aa010197c040cfcebe0",
-                "workload": "small", "bytes_per_launch": 187561984 + 42736896,
+ATTN_TRAFFIC = {"sha256_rf_attn_cu": "c67d094926473c0d583bbae9999411ba0928f87ed1503a6888e306c8abd315d0",
+                "workload": "small", "bytes_per_launch": 188244224 + 47994624,
                 "launch": "schedule step 0 of the small workload (all 13 frames active)"}
 
 
@@ -229,6 +229,7 @@ def run_gpu(args):
     if ATTN_TRAFFIC["sha256_rf_attn_cu"] == _sha(attn_src) and args.config == ATTN_TRAFFIC["workload"]:
         traffic = ATTN_TRAFFIC["bytes_per_launch"]
     bw = run_bandwidth(w, dev, peaks) if not args.no_bandwidth else None
+    sweep = run_sweep(w, dev, Q, K, V, O, vel, max(3, min(K_steps, 10))) if w.sweep else None
     status = int(core.status.item()) | int(core_all.status.item())
 
     out = {
@@ -261,6 +262,7 @@ def run_gpu(args):
             "avg_launch_ms": round(attn_ms_total / len(ev), 5),
         },
         "bandwidth_kernels": bw,
+        "active_fraction_sweep": sweep,
         "e2e": e2e,
         "gpu_launches": 4 * K_steps,
         "clocks": clocks,
@@ -352,10 +354,21 @@ def run_bandwidth(w, dev, peaks):
     A = int(p["mask"][s].sum())
     bytes_project = (12 * (F - A) + 8 * A) * E
     bytes_step = 12 * A * E
+    # the all-frames-active step for the Euler update as well (largest launch)
+    mask0 = torch.from_numpy(p["mask"][0]).to(dev)
+    act0 = torch.zeros(F, dtype=torch.int32, device=dev)
+    cnt0 = torch.zeros(2, dtype=torch.int32, device=dev)
+    rf.rf_schedule_compact(mask0, F, w.N, act0, skp, None, cnt0)
+    dt0 = torch.from_numpy(p["dt"][0]).to(dev)
+    slot0 = torch.from_numpy(p["cur_slot"][0]).to(dev)
+    A0 = int(p["mask"][0].sum())
     res = {}
-    for name, fn, nbytes in (
-            ("rf_project", lambda: rf.rf_project(ctx, z2, slot, alpha, beta, F, E), bytes_project),
-            ("rf_step", lambda: rf.rf_step(z2, slot, v, dt, act, cnt, F, E), bytes_step)):
+    for name, fn, nbytes, step, nact in (
+            ("rf_project", lambda: rf.rf_project(ctx, z2, slot, alpha, beta, F, E), bytes_project,
+             s, A),
+            ("rf_step", lambda: rf.rf_step(z2, slot, v, dt, act, cnt, F, E), bytes_step, s, A),
+            ("rf_step_all_active", lambda: rf.rf_step(z2, slot0, v, dt0, act0, cnt0, F, E),
+             12 * A0 * E, 0, A0)):
         times = []
         for rep in range(13):
             flush.fill_(rep)
@@ -371,10 +384,53 @@ def run_bandwidth(w, dev, peaks):
         gbs = nbytes / (ms * 1e-3) / 1e9
         res[name] = {"GB/s": round(gbs, 1), "frac": round(gbs / peaks["hbm_gbs"], 4),
                      "peak": peaks["hbm_gbs"], "ms": round(ms, 4), "bytes": nbytes,
-                     "shape": f"F={F} x E={E} fp32 (C = H*d = {w.H * w.d}), step {s}, A={A}"}
+                     "shape": f"F={F} x E={E} fp32 (C = H*d = {w.H * w.d}), step {step}, "
+                              f"A={nact}"}
     del z2, ctx, v, flush
     torch.cuda.empty_cache()
     return res
+
+
+def run_sweep(w, dev, Q, K, V, O, vel, steps):
+    """Step core with a fixed active-frame mask for each active fraction of the workload
+    (frames {floor(i*F/A)}), against the all-frames-active step."""
+    import numpy as np
+    import torch
+    import workloads as wl
+    from paper_2606_06309_gb300.stepcore import Plan, StepCore
+    E = w.N * w.C
+    out = {"fractions": [], "active_frames": [], "step_core_ms": [], "attn_tflops": []}
+    for frac, mask in zip(w.sweep, wl.sweep_masks(w.F, w.sweep)):
+        m = np.tile(np.asarray(mask, np.uint8), (w.S, 1))
+        alpha = np.where(m == 1, 1.0, 0.5).astype(np.float32)
+        host = {"mask": m, "alpha": alpha, "beta": (1 - alpha).astype(np.float32),
+                "dt": np.where(m == 1, -1.0 / w.S, 0.0).astype(np.float32),
+                "cur_slot": np.zeros_like(m)}
+        t = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
+        plan = Plan(t["mask"], t["alpha"], t["beta"], t["dt"], t["cur_slot"], host)
+        core = StepCore(w.F, w.N, E, w.H, w.d, plan, dev)
+        for k in range(3):
+            core.run(k % w.S, vel[k % w.S], O, Q, K, V, w.softmax_scale)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for k in range(steps):
+            core.run(k % w.S, vel[k % w.S], O, Q, K, V, w.softmax_scale)
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / steps
+        A = int(sum(mask))
+        out["fractions"].append(frac)
+        out["active_frames"].append(A)
+        out["step_core_ms"].append(round(ms, 4))
+        out["attn_tflops"].append(round(4 * A * w.N * w.S_tok * w.d * w.H / (ms * 1e-3) / 1e12, 1))
+        assert core.status.item() == 0
+    dense = out["step_core_ms"][out["fractions"].index(1.0)] if 1.0 in out["fractions"] else None
+    if dense:
+        out["speedup_vs_all_active"] = [round(dense / x, 3) for x in out["step_core_ms"]]
+        out["ideal_speedup"] = [round(w.F / A, 3) for A in out["active_frames"]]
+    return out
 
 
 # ---------------------------------------------------------------------------

@@ -146,47 +146,50 @@ __global__ void __launch_bounds__(kStreamThreads)
   }
 }
 
+// Euler step over the active frames only.  The active count lives on the device, so the grid
+// is fixed (a few waves) and walks (active frame, chunk of kStreamThreads*kUnroll float4s)
+// pairs with a stride of gridDim.x chunks: the work spreads over every SM whatever A is.
 __global__ void __launch_bounds__(kStreamThreads)
     step_kernel(float4* __restrict__ z2, const uint8_t* __restrict__ cur_slot,
                 const float4* __restrict__ vel, const float* __restrict__ dt,
                 const int32_t* __restrict__ active, const int32_t* __restrict__ counts, int F,
                 int64_t E4) {
-  const int slot_idx = blockIdx.y;
-  if (slot_idx >= counts[0]) return;
-  const int f = active[slot_idx];
-  if (f < 0 || f >= F) return;
-  const int c = cur_slot[f] & 1;
-  const float h = dt[f];
-  const float4* z = z2 + (static_cast<int64_t>(c) * F + f) * E4;
-  float4* out = z2 + (static_cast<int64_t>(c ^ 1) * F + f) * E4;
-  const float4* v = vel + static_cast<int64_t>(f) * E4;
-  const int64_t step = static_cast<int64_t>(gridDim.x) * kStreamThreads;
-  int64_t i = static_cast<int64_t>(blockIdx.x) * kStreamThreads + threadIdx.x;
-  for (; i + (kUnroll - 1) * step < E4; i += kUnroll * step) {
+  constexpr int64_t kChunk = static_cast<int64_t>(kStreamThreads) * kUnroll;
+  int A = counts[0];
+  A = A < 0 ? 0 : (A > F ? F : A);
+  const int64_t per_frame = (E4 + kChunk - 1) / kChunk;
+  const int64_t total = per_frame * A;
+  for (int64_t c = blockIdx.x; c < total; c += gridDim.x) {
+    const int a = static_cast<int>(c / per_frame);
+    const int64_t base = (c - a * per_frame) * kChunk + threadIdx.x;
+    const int f = active[a];
+    if (f < 0 || f >= F) continue;
+    const int sl = cur_slot[f] & 1;
+    const float h = dt[f];
+    const float4* z = z2 + (static_cast<int64_t>(sl) * F + f) * E4;
+    float4* out = z2 + (static_cast<int64_t>(sl ^ 1) * F + f) * E4;
+    const float4* v = vel + static_cast<int64_t>(f) * E4;
     float4 x[kUnroll], y[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      x[u] = ld_stream(z + i + u * step);
-      y[u] = ld_stream(v + i + u * step);
+      const int64_t i = base + u * kStreamThreads;
+      if (i < E4) {
+        x[u] = ld_stream(z + i);
+        y[u] = ld_stream(v + i);
+      }
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
-      float4 r;
-      r.x = fmaf(h, y[u].x, x[u].x);
-      r.y = fmaf(h, y[u].y, x[u].y);
-      r.z = fmaf(h, y[u].z, x[u].z);
-      r.w = fmaf(h, y[u].w, x[u].w);
-      st_stream(out + i + u * step, r);
+      const int64_t i = base + u * kStreamThreads;
+      if (i < E4) {
+        float4 r;
+        r.x = fmaf(h, y[u].x, x[u].x);
+        r.y = fmaf(h, y[u].y, x[u].y);
+        r.z = fmaf(h, y[u].z, x[u].z);
+        r.w = fmaf(h, y[u].w, x[u].w);
+        st_stream(out + i, r);
+      }
     }
-  }
-  for (; i < E4; i += step) {
-    const float4 x = ld_stream(z + i), y = ld_stream(v + i);
-    float4 r;
-    r.x = fmaf(h, y.x, x.x);
-    r.y = fmaf(h, y.y, x.y);
-    r.z = fmaf(h, y.z, x.z);
-    r.w = fmaf(h, y.w, x.w);
-    st_stream(out + i, r);
   }
 }
 
@@ -256,8 +259,12 @@ extern "C" rf_status rf_step(float* d_z2, const uint8_t* d_cur_slot, const float
   DeviceInfo di;
   if (rf_status st = current_device_info(&di)) return st;
   const int64_t E4 = E / 4;
-  dim3 grid(blocks_per_frame(E4, di.sm_count), F);
-  step_kernel<<<grid, kStreamThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+  // enough chunks in flight to cover every SM a few times, never more than the largest A needs
+  const int64_t chunk = static_cast<int64_t>(kStreamThreads) * kUnroll;
+  int64_t blocks = ((E4 + chunk - 1) / chunk) * F;
+  if (blocks > 8LL * di.sm_count) blocks = 8LL * di.sm_count;
+  step_kernel<<<static_cast<int>(blocks), kStreamThreads, 0,
+                reinterpret_cast<cudaStream_t>(stream)>>>(
       reinterpret_cast<float4*>(d_z2), d_cur_slot, reinterpret_cast<const float4*>(d_v), d_dt,
       d_active, d_counts, F, E4);
   return launch_status("step_kernel launch");
