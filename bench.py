@@ -119,6 +119,21 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
+def combine_ranks(ms_local: float, flops_local: float, dist=None, device="cpu"):
+    """Whole-job throughput of N replicas: the slowest rank's time (all ranks start together
+    after a barrier) and every rank's FLOPs.  Returns (max_ms, total_flops, TFLOP/s)."""
+    import torch
+    t = torch.tensor([ms_local, flops_local], dtype=torch.float64, device=device)
+    if dist is not None and dist.is_initialized() and dist.get_world_size() > 1:
+        ms_t = t[:1].clone()
+        fl_t = t[1:].clone()
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+        dist.all_reduce(fl_t, op=dist.ReduceOp.SUM)
+        t = torch.cat([ms_t, fl_t])
+    max_ms, total = float(t[0].item()), float(t[1].item())
+    return max_ms, total, total / (max_ms * 1e-3) / 1e12
+
+
 def _gpu_index(local_rank):
     vis = os.environ.get("CUDA_VISIBLE_DEVICES")
     if vis:
@@ -202,13 +217,9 @@ def run_gpu(args):
     with ClockSampler(_gpu_index(local)) as clk:
         ms, _ = timed(core, K_steps, W_steps)
     clocks = clk.summary()
-    # max over ranks
-    ms_t = torch.tensor([ms], device=dev, dtype=torch.float64)
-    if dist is not None:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
-    total_flops = sum(flops_step[k % S] for k in range(K_steps)) * world
-    value = total_flops / (ms * 1e-3) / 1e12
+    # slowest rank's time, every rank's work
+    ms, total_flops, value = combine_ranks(
+        ms, float(sum(flops_step[k % S] for k in range(K_steps))), dist, dev)
 
     # per-launch attention timing for the roofline (separate pass, same work)
     _, ev = timed(core, K_steps, 0, per_launch=True)
@@ -311,12 +322,9 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
         one(k)
     t1.record(stream)
     barrier()
-    ms = t0.elapsed_time(t1)
-    ms_t = torch.tensor([ms], device=Q.device, dtype=torch.float64)
-    if dist is not None:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms = float(ms_t.item())
-    flops = sum(flops_step[k % S] for k in range(K_steps)) * world
+    ms, flops, _ = combine_ranks(t0.elapsed_time(t1),
+                                 float(sum(flops_step[k % S] for k in range(K_steps))), dist,
+                                 Q.device)
     h2d = 3 * Q.numel() * Q.element_size() + vel[0].numel() * 4
     d2h = Q.numel() * Q.element_size() + core.z2.numel() * 4
     return {"value": round(flops / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "steps": K_steps,

@@ -229,6 +229,21 @@ rf_status rf_step(float* d_z2, const uint8_t* d_cur_slot, const float* d_v, cons
                   const int32_t* d_active, const int32_t* d_counts, int F, int64_t E,
                   rf_stream_t stream);
 
+/*
+ * rf_selftest_bounded_wait -- check, on the GPU, the path every device-side wait
+ * of rf_attn takes when it runs out of time.  No paper passage: this is a
+ * failure-handling self-test.
+ *
+ * Launches one CTA that allocates tensor memory, waits on an mbarrier that
+ * nothing ever arrives at, gives up after limit_us microseconds
+ * (100 <= limit_us <= 2,000,000), ORs RF_ERR_DEVICE_TIMEOUT into *d_status,
+ * frees its tensor memory and returns.  Nothing faults or traps and the context
+ * stays usable.  The caller zeroes *d_status first and reads it after
+ * synchronising.  Returns RF_ERR_INVALID_ARG for a null pointer or an out-of-range
+ * limit.
+ */
+rf_status rf_selftest_bounded_wait(int32_t* d_status, int limit_us, rf_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -25,7 +25,7 @@ _LIB: Optional[ctypes.CDLL] = None
 # Every symbol include/rf.h declares.
 EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
            "rf_schedule_compact", "rf_project", "rf_attn", "rf_attn_workspace_bytes",
-           "rf_attn_noalloc", "rf_step")
+           "rf_attn_noalloc", "rf_step", "rf_selftest_bounded_wait")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
 _SIG = {
@@ -38,6 +38,7 @@ _SIG = {
     "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
                  _vp, _i64, _vp, _vp], _i32),
     "rf_attn_workspace_bytes": ([_i32], _i64),
+    "rf_selftest_bounded_wait": ([_vp, _i32, _vp], _i32),
     "rf_attn_noalloc": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
                          _f32, _vp, _vp], _i32),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
@@ -148,6 +149,12 @@ def rf_attn_noalloc(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: 
     _check("rf_attn_noalloc", load().rf_attn_noalloc(
         _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
         _ptr(active), _ptr(counts), float(softmax_scale), _ptr(status), _stream(stream)))
+
+
+def rf_selftest_bounded_wait(status, limit_us: int, stream=None):
+    """Run the device bounded-wait self-test; *status receives RF_ERR_DEVICE_TIMEOUT."""
+    _check("rf_selftest_bounded_wait", load().rf_selftest_bounded_wait(
+        _ptr(status), int(limit_us), _stream(stream)))
 
 
 def rf_attn_workspace_bytes(d: int) -> int:

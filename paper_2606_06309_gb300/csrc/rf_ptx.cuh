@@ -45,17 +45,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Wait until the phase with the given parity of barrier `bar` has completed.
 // Gives up after `limit_ns` of wall-clock time or as soon as another thread of the CTA has
-// raised *abort; on expiry it raises *abort itself.  Returns false when it gave up.
+// raised *abort; on expiry it raises *abort itself.  Returns false when it gave up.  A spin
+// count (limit_ns / 16 rounds of 32 polls, far more than the time limit allows) bounds the
+// loop even if the timer did not advance.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort,
                                           uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
-  while (true) {
+  const uint64_t max_rounds = limit_ns >> 4;
+  for (uint64_t n = 0;; ++n) {
 #pragma unroll 1
     for (int i = 0; i < 32; ++i)
       if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (globaltimer_ns() - t0 > limit_ns) {
+    if (n >= max_rounds || globaltimer_ns() - t0 > limit_ns) {
       *abort = 1;
       return false;
     }

@@ -1,0 +1,51 @@
+"""The N > 1 path of bench.py on the CPU: N independent replicas, one per rank.
+
+Whole-job throughput is every rank's FLOPs over the slowest rank's time (max over ranks).
+These tests run two gloo ranks on the CPU; no GPU and no collective on the data path."""
+import os
+import subprocess
+import sys
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    sys.path.insert(0, ROOT)
+    import bench
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        ms_local = [2.0, 3.0][rank]        # rank 1 is the slower replica
+        flops_local = [1e12, 1e12][rank]
+        out[rank] = bench.combine_ranks(ms_local, flops_local, dist)
+    finally:
+        dist.destroy_process_group()
+
+
+def test_combine_ranks_gloo_world2():
+    port = 29500 + os.getpid() % 1000
+    out = mp.Manager().dict()
+    mp.spawn(_worker, args=(2, port, out), nprocs=2, join=True)
+    for r in range(2):
+        max_ms, total, tflops = out[r]
+        assert max_ms == 3.0 and total == 2e12
+        assert tflops == pytest.approx(2e12 / 3e-3 / 1e12)
+
+
+def test_combine_ranks_single_process():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.combine_ranks(4.0, 8e12) == (4.0, 8e12, pytest.approx(2000.0))
+
+
+def test_reference_arm_nonzero_rank_exits_without_work():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--config", "tiny", "--steps", "1", "--warmup", "0"],
+                       capture_output=True, text=True, env=env, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip() == ""
