@@ -96,3 +96,71 @@ class StepCore:
         self.project(s, stream)
         self.attn(O, Q, K, V, scale, lse, stream)
         self.step(s, v, stream)
+
+
+class HostPipeline:
+    """Step-core steps fed from pinned host memory, with the copies hidden behind compute.
+
+    Each step's inputs (Q, K, V and the velocity) are copied host -> device and its results
+    (the attention output O and a snapshot of the two-slot latent store) device -> host.  Two
+    device buffer sets and two copy streams (one per direction, so both copy engines work)
+    overlap the input copy of step k+1 and the read-back of step k-1 with the compute of
+    step k.  Events order the three streams; nothing synchronises the host.
+    """
+
+    def __init__(self, core: StepCore, S_tok: int, device="cuda"):
+        dev = torch.device(device)
+        self.core = core
+        self.compute = torch.cuda.current_stream(dev)
+        self.h2d = torch.cuda.Stream(dev)
+        self.d2h = torch.cuda.Stream(dev)
+        H, d, F, E = core.H, core.d, core.F, core.E
+        self.buf = []
+        for _ in range(2):
+            self.buf.append({
+                "Q": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
+                "K": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
+                "V": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
+                "v": torch.empty(F, E, dtype=torch.float32, device=dev),
+                "O": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
+                "z": torch.empty(2, F, E, dtype=torch.float32, device=dev),
+            })
+        ev = lambda: torch.cuda.Event()
+        self.loaded = [ev(), ev()]     # inputs of buffer b are on the device
+        self.consumed = [ev(), ev()]   # compute finished with buffer b (inputs read, outputs ready)
+        self.drained = [ev(), ev()]    # outputs of buffer b are back on the host
+        self.k = 0
+
+    def step(self, s: int, hQ, hK, hV, hv, hO, hz, scale: float):
+        """Enqueue schedule step s: inputs from pinned host tensors hQ, hK, hV (bf16
+        [S_tok, H, d]) and hv (fp32 [F, E]); results into pinned hO (bf16) and hz (fp32
+        [2, F, E]).  Returns immediately."""
+        b = self.k % 2
+        B = self.buf[b]
+        first_use = self.k < 2
+        with torch.cuda.stream(self.h2d):
+            if not first_use:
+                self.h2d.wait_event(self.consumed[b])   # step k-2 has read these inputs
+            B["Q"].copy_(hQ, non_blocking=True)
+            B["K"].copy_(hK, non_blocking=True)
+            B["V"].copy_(hV, non_blocking=True)
+            B["v"].copy_(hv, non_blocking=True)
+            self.loaded[b].record(self.h2d)
+        self.compute.wait_event(self.loaded[b])
+        if not first_use:
+            self.compute.wait_event(self.drained[b])    # step k-2's outputs are on the host
+        self.core.run(s, B["v"], B["O"], B["Q"], B["K"], B["V"], scale, stream=self.compute)
+        B["z"].copy_(self.core.z2, non_blocking=True)
+        self.consumed[b].record(self.compute)
+        with torch.cuda.stream(self.d2h):
+            self.d2h.wait_event(self.consumed[b])
+            hO.copy_(B["O"], non_blocking=True)
+            hz.copy_(B["z"], non_blocking=True)
+            self.drained[b].record(self.d2h)
+        self.k += 1
+
+    def bytes_per_step(self):
+        B = self.buf[0]
+        h2d = sum(B[n].numel() * B[n].element_size() for n in ("Q", "K", "V", "v"))
+        d2h = sum(B[n].numel() * B[n].element_size() for n in ("O", "z"))
+        return h2d, d2h
