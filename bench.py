@@ -360,8 +360,17 @@ def run_bandwidth(w, dev, peaks):
     dt0 = torch.from_numpy(p["dt"][0]).to(dev)
     slot0 = torch.from_numpy(p["cur_slot"][0]).to(dev)
     A0 = int(p["mask"][0].sum())
+    # rolling key/value cache: bf16 K/V rows [S_tok][H*d] and two-slot caches [2][F][N][H*d]
+    D = w.H * w.d
+    Kb = torch.randn(F * w.N, D, device=dev).to(torch.bfloat16)
+    Vb = torch.randn(F * w.N, D, device=dev).to(torch.bfloat16)
+    Kc = torch.randn(2, F, w.N, D, device=dev).to(torch.bfloat16)
+    Vc = torch.randn(2, F, w.N, D, device=dev).to(torch.bfloat16)
+    bytes_kv = 2 * (6 * (F - A) + 4 * A) * w.N * D
     res = {}
     for name, fn, nbytes, step, nact in (
+            ("rf_project_kv", lambda: rf.rf_project_kv(Kb, Vb, D, Kc, Vc, slot, alpha, beta, act,
+                                                       skp, cnt, F, w.N, D), bytes_kv, s, A),
             ("rf_project", lambda: rf.rf_project(ctx, z2, slot, alpha, beta, F, E), bytes_project,
              s, A),
             ("rf_step", lambda: rf.rf_step(z2, slot, v, dt, act, cnt, F, E), bytes_step, s, A),
@@ -384,7 +393,9 @@ def run_bandwidth(w, dev, peaks):
                      "peak": peaks["hbm_gbs"], "ms": round(ms, 4), "bytes": nbytes,
                      "shape": f"F={F} x E={E} fp32 (C = H*d = {w.H * w.d}), step {step}, "
                               f"A={nact}"}
-    del z2, ctx, v, flush
+    res["rf_project_kv"]["shape"] = (f"K and V bf16 [{F * w.N}][{D}] + caches [2][{F}][{w.N}]"
+                                     f"[{D}], step {s}, A={A}")
+    del z2, ctx, v, flush, Kb, Vb, Kc, Vc
     torch.cuda.empty_cache()
     return res
 
@@ -510,11 +521,20 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bandwidth", action="store_true")
+    ap.add_argument("--bandwidth-only", action="store_true",
+                    help="only the bandwidth-kernel leg (for profiling); prints its JSON")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl != "reference":
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.bandwidth_only:
+        import torch
+        import workloads as wl
+        import paper_2606_06309_gb300 as rf
+        rf.load()
+        peaks, _ = _peaks()
+        print(json.dumps(run_bandwidth(wl.get(args.config), torch.device("cuda", 0), peaks)))
     else:
         run_gpu(args)
 

@@ -135,6 +135,29 @@ rf_status rf_project(float* d_ctx, const float* d_z2, const uint8_t* d_cur_slot,
                      rf_stream_t stream);
 
 /*
+ * rf_project_kv -- per-layer rolling key/value cache (Appendix B.2), one layer, one
+ * step, keys and values together.
+ *
+ *   d_K, d_V     bf16 attention inputs, row t = token at base + t*kv_row_stride,
+ *                D contiguous elements (D = H*d, heads interleaved)
+ *   d_Kc, d_Vc   bf16 two-slot caches [2][F][N][D] (slot cur_slot[f] = the frame's latest
+ *                cached state "after", the other slot the state before it)
+ *   d_cur_slot, d_alpha, d_beta  [F] this step's slot bits and Eq. 3 weights (the plan)
+ *   d_active, d_skipped, d_counts  lists from rf_schedule_compact (device)
+ *   F, N, D      frames, tokens per frame, elements per token (D % 8 == 0,
+ *                kv_row_stride % 8 == 0, all bases 16-byte aligned)
+ * For each skipped frame f its K and V rows are overwritten with
+ *   bf16(fmaf(alpha[f], after, beta[f] * before))        (fp32 arithmetic, RNE)
+ * and for each active frame its fresh K and V rows are copied into the cache's other
+ * slot (the plan's slot flip then makes them "after": shift-and-store).  Rows of
+ * active frames and caches of skipped frames are not written.  One launch.
+ */
+rf_status rf_project_kv(void* d_K, void* d_V, int64_t kv_row_stride, void* d_Kc, void* d_Vc,
+                        const uint8_t* d_cur_slot, const float* d_alpha, const float* d_beta,
+                        const int32_t* d_active, const int32_t* d_skipped,
+                        const int32_t* d_counts, int F, int N, int D, rf_stream_t stream);
+
+/*
  * rf_attn -- active-query x full-sequence softmax attention (Sec. 3.2.4 and
  * Appendix B.2: the active frames' queries attend to the keys and values of
  * all F*N tokens, true for active frames and projected for skipped ones).

@@ -18,6 +18,9 @@ Citations name the paper's sections, equations and algorithms:
                        attention in fp64, brute force over every key.
 * euler()           -- the heterogeneous update of Algorithm 2 / Sec. 3.2.3 as a
                        rectified-flow Euler step z <- z + (sigma_to - sigma_from) v.
+* project_kv_cache() -- Appendix B.2, per-layer rolling cache: skipped frames'
+                       keys/values projected with Eq. 3 from the two cached states,
+                       active frames' fresh keys/values shifted into the cache.
 * keyframe_select() -- Algorithm 1 (dynamic sequential keyframe selection),
                        Eq. 1.  Parity partly unpinned: the paper gives no values
                        for tau, delta tau, delta_up, delta_down.
@@ -32,7 +35,7 @@ from typing import Dict, Optional, Sequence
 import numpy as np
 
 __all__ = ["sigmas", "schedule", "active_set_alg2", "compact", "project", "attention",
-           "euler", "sampler", "flops_attn", "keyframe_select", "to_f64"]
+           "euler", "sampler", "flops_attn", "keyframe_select", "project_kv_cache", "to_f64"]
 
 
 def to_f64(x) -> np.ndarray:
@@ -184,6 +187,31 @@ def attention(Q, K, V, rows: Sequence[int], scale: float, heads: Optional[Sequen
             O[c0:c0 + chunk, hi, :] = (e @ Vh) / l
             L[hi, c0:c0 + chunk] = (m + np.log(l))[:, 0]
     return O, L
+
+
+def project_kv_cache(KV, cache, cur_slot, alpha, mask):
+    """Per-layer rolling cache of Appendix B.2 for one key or value tensor.
+
+    KV: [F, N, D] the step's keys (or values): rows of active frames are fresh.
+    cache: [2, F, N, D] two cached states per frame; slot cur_slot[f] holds the frame's
+    latest state ("after"), the other slot the one before it ("before").
+    alpha: [F] projection weights of the step; mask: [F] 1 = active.
+    Skipped frame: its rows become (1 - alpha) * before + alpha * after (Eq. 3 with the
+    cache's two states and the step's weight).  Active frame: its fresh rows are stored as
+    the new "after" (into the other slot; the slot flip of the plan makes the old "after"
+    the new "before": shift-and-store).
+    Returns (KV_out [F, N, D], cache_out [2, F, N, D]) in fp64.
+    """
+    kv = to_f64(KV).copy()
+    c = to_f64(cache).copy()
+    for f in range(kv.shape[0]):
+        cur = int(cur_slot[f])
+        if mask[f]:
+            c[1 - cur, f] = kv[f]
+        else:
+            a = float(alpha[f])
+            kv[f] = (1.0 - a) * c[1 - cur, f] + a * c[cur, f]
+    return kv, c
 
 
 def euler(z, v, dt) -> np.ndarray:

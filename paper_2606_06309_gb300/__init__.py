@@ -15,7 +15,7 @@ from typing import Optional
 import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_attn", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
+           "rf_project", "rf_project_kv", "rf_attn", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
            "rf_status_str",
            "rf_version", "EXPORTS"]
 
@@ -24,7 +24,8 @@ _LIB: Optional[ctypes.CDLL] = None
 
 # Every symbol include/rf.h declares.
 EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
-           "rf_schedule_compact", "rf_project", "rf_attn", "rf_attn_workspace_bytes",
+           "rf_schedule_compact", "rf_project", "rf_project_kv", "rf_attn",
+           "rf_attn_workspace_bytes",
            "rf_attn_noalloc", "rf_step", "rf_selftest_bounded_wait")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
@@ -35,6 +36,8 @@ _SIG = {
     "rf_plan_build": ([_i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp], _i32),
     "rf_schedule_compact": ([_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp], _i32),
     "rf_project": ([_vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
+    "rf_project_kv": ([_vp, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _i32, _i32,
+                       _vp], _i32),
     "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
                  _vp, _i64, _vp, _vp], _i32),
     "rf_attn_workspace_bytes": ([_i32], _i64),
@@ -130,6 +133,13 @@ def rf_schedule_compact(mask, F: int, N: int, active, skipped, token_idx, counts
 def rf_project(ctx, z2, cur_slot, alpha, beta, F: int, E: int, stream=None):
     _check("rf_project", load().rf_project(
         _ptr(ctx), _ptr(z2), _ptr(cur_slot), _ptr(alpha), _ptr(beta), F, E, _stream(stream)))
+
+
+def rf_project_kv(K, V, kv_row_stride: int, Kc, Vc, cur_slot, alpha, beta, active, skipped,
+                  counts, F: int, N: int, D: int, stream=None):
+    _check("rf_project_kv", load().rf_project_kv(
+        _ptr(K), _ptr(V), kv_row_stride, _ptr(Kc), _ptr(Vc), _ptr(cur_slot), _ptr(alpha),
+        _ptr(beta), _ptr(active), _ptr(skipped), _ptr(counts), F, N, D, _stream(stream)))
 
 
 def rf_attn(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: int, H: int,

@@ -1,6 +1,7 @@
 // rf_stream.cu -- the bandwidth kernels of the step core:
 //   rf_schedule_compact  active-frame mask -> index lists (warp ballot / popc scan)
 //   rf_project           Eq. 3 latent trajectory projection (128-bit streaming)
+//   rf_project_kv        rolling key/value cache of Appendix B.2 (bf16, 128-bit streaming)
 //   rf_step              Euler update of the active frames (128-bit streaming)
 #include <cuda_runtime.h>
 
@@ -193,6 +194,111 @@ __global__ void __launch_bounds__(kStreamThreads)
   }
 }
 
+// ---------------------------------------------------------------------------------------
+// Rolling key/value cache (Appendix B.2).  blockIdx.y selects keys or values.  The grid walks
+// (frame-list index, chunk) pairs over all F frames: list index a < A is the active frame
+// active[a], whose fresh rows are stored into its cache's other slot (shift-and-store); the
+// rest are skipped[a - A], whose rows are rewritten with Eq. 3 from the two cached states.
+// Eight bf16 per 16-byte access; fp32 arithmetic, rounded to nearest even.
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t proj_pair(uint32_t cur, uint32_t prev, float a, float b) {
+  const float lo = fmaf(a, bf16_lo(cur), b * bf16_lo(prev));
+  const float hi = fmaf(a, bf16_hi(cur), b * bf16_hi(prev));
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__global__ void __launch_bounds__(kStreamThreads)
+    project_kv_kernel(uint16_t* __restrict__ K, uint16_t* __restrict__ V, int64_t row_stride,
+                      uint16_t* __restrict__ Kc, uint16_t* __restrict__ Vc,
+                      const uint8_t* __restrict__ cur_slot, const float* __restrict__ alpha,
+                      const float* __restrict__ beta, const int32_t* __restrict__ active,
+                      const int32_t* __restrict__ skipped, const int32_t* __restrict__ counts,
+                      int F, int N, int D) {
+  uint16_t* X = blockIdx.y ? V : K;
+  uint16_t* Xc = blockIdx.y ? Vc : Kc;
+  int A = counts[0];
+  A = A < 0 ? 0 : (A > F ? F : A);
+  const int D8 = D >> 3;                      // 16-byte vectors per row
+  const int64_t frame_vecs = static_cast<int64_t>(N) * D8;
+  constexpr int64_t kChunk = static_cast<int64_t>(kStreamThreads) * kUnroll;
+  const int64_t per_frame = (frame_vecs + kChunk - 1) / kChunk;
+  const int64_t total = per_frame * F;
+  const int64_t slot_stride = static_cast<int64_t>(F) * N * D;  // elements between slots
+  const bool contiguous = row_stride == D;  // K/V rows back to back: no row arithmetic
+  for (int64_t c = blockIdx.x; c < total; c += gridDim.x) {
+    const int a = static_cast<int>(c / per_frame);
+    const int64_t base = (c - a * per_frame) * kChunk + threadIdx.x;
+    const bool is_active = a < A;
+    const int f = is_active ? active[a] : skipped[a - A];
+    if (f < 0 || f >= F) continue;
+    const int sl = cur_slot[f] & 1;
+    const uint4* cur = reinterpret_cast<const uint4*>(Xc + sl * slot_stride +
+                                                      static_cast<int64_t>(f) * N * D);
+    uint4* prev = reinterpret_cast<uint4*>(Xc + (sl ^ 1) * slot_stride +
+                                           static_cast<int64_t>(f) * N * D);
+    uint16_t* rows = X + static_cast<int64_t>(f) * N * row_stride;
+    // vector index of the k-th vector of this thread inside the frame's K/V rows: (row, col)
+    // advanced incrementally (one division per chunk, none per vector)
+    int64_t off[kUnroll];
+    {
+      int64_t p = 0, q = base;
+      if (!contiguous) {
+        p = static_cast<uint32_t>(base) / static_cast<uint32_t>(D8);  // < 2^31 (host check)
+        q = base - p * D8;
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        off[u] = contiguous ? base + u * kStreamThreads : p * (row_stride >> 3) + q;
+        if (!contiguous) {
+          q += kStreamThreads;
+          while (q >= D8) {
+            q -= D8;
+            ++p;
+          }
+        }
+      }
+    }
+    uint4* rv = reinterpret_cast<uint4*>(rows);
+    if (is_active) {
+      uint4 x[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u)
+        if (base + u * kStreamThreads < frame_vecs) x[u] = __ldcs(rv + off[u]);
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t v = base + u * kStreamThreads;
+        if (v < frame_vecs) __stcs(prev + v, x[u]);  // the other slot
+      }
+    } else {
+      const float al = alpha[f], be = beta[f];
+      uint4 x[kUnroll], y[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t v = base + u * kStreamThreads;
+        if (v < frame_vecs) {
+          x[u] = __ldcs(cur + v);
+          y[u] = __ldcs(prev + v);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        if (base + u * kStreamThreads < frame_vecs) {
+          uint4 r;
+          r.x = proj_pair(x[u].x, y[u].x, al, be);
+          r.y = proj_pair(x[u].y, y[u].y, al, be);
+          r.z = proj_pair(x[u].z, y[u].z, al, be);
+          r.w = proj_pair(x[u].w, y[u].w, al, be);
+          __stcs(rv + off[u], r);
+        }
+      }
+    }
+  }
+}
+
 // Blocks per frame so that the whole grid covers a few waves of the device even when only
 // one frame is active, without launching blocks that would have nothing to do.
 int blocks_per_frame(int64_t E4, int sm_count) {
@@ -268,4 +374,32 @@ extern "C" rf_status rf_step(float* d_z2, const uint8_t* d_cur_slot, const float
       reinterpret_cast<float4*>(d_z2), d_cur_slot, reinterpret_cast<const float4*>(d_v), d_dt,
       d_active, d_counts, F, E4);
   return launch_status("step_kernel launch");
+}
+
+extern "C" rf_status rf_project_kv(void* d_K, void* d_V, int64_t kv_row_stride, void* d_Kc,
+                                   void* d_Vc, const uint8_t* d_cur_slot, const float* d_alpha,
+                                   const float* d_beta, const int32_t* d_active,
+                                   const int32_t* d_skipped, const int32_t* d_counts, int F,
+                                   int N, int D, rf_stream_t stream) {
+  if (!d_K || !d_V || !d_Kc || !d_Vc || !d_cur_slot || !d_alpha || !d_beta || !d_active ||
+      !d_skipped || !d_counts)
+    return RF_ERR_INVALID_ARG;
+  if (F < 1 || F > kMaxFrames || N < 1 || D < 8) return RF_ERR_INVALID_ARG;
+  if (kv_row_stride < D) return RF_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(N) * (D / 8) > 0x7FFFFFFF) return RF_ERR_INVALID_ARG;
+  if (D % 8 != 0 || kv_row_stride % 8 != 0) return RF_ERR_MISALIGNED;
+  if (!aligned16(d_K) || !aligned16(d_V) || !aligned16(d_Kc) || !aligned16(d_Vc))
+    return RF_ERR_MISALIGNED;
+  DeviceInfo di;
+  if (rf_status st = current_device_info(&di)) return st;
+  const int64_t frame_vecs = static_cast<int64_t>(N) * (D / 8);
+  const int64_t chunk = static_cast<int64_t>(kStreamThreads) * kUnroll;
+  int64_t blocks = ((frame_vecs + chunk - 1) / chunk) * F;
+  if (blocks > 4LL * di.sm_count) blocks = 4LL * di.sm_count;
+  dim3 grid(static_cast<unsigned>(blocks), 2);
+  project_kv_kernel<<<grid, kStreamThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      static_cast<uint16_t*>(d_K), static_cast<uint16_t*>(d_V), kv_row_stride,
+      static_cast<uint16_t*>(d_Kc), static_cast<uint16_t*>(d_Vc), d_cur_slot, d_alpha, d_beta,
+      d_active, d_skipped, d_counts, F, N, D);
+  return launch_status("project_kv_kernel launch");
 }

@@ -386,3 +386,90 @@ def test_host_pipeline_matches_device_path(cuda_lib, name):
         assert torch.equal(hO[s][act], outs[s][0][act]), s
         assert torch.equal(hz[s], outs[s][1]), s
     assert core.status.item() == 0
+
+
+# ---------------------------------------------------------------------------
+# rf_project_kv: rolling key/value cache (Appendix B.2)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("F,N,H,d,fused", [
+    (5, 64, 2, 64, False),
+    (7, 1560, 12, 128, False),
+    (4, 200, 3, 128, True),   # K, V slices of a fused [tokens, 3, H, d] buffer
+    (1, 8, 1, 64, False),
+])
+def test_project_kv_parity(cuda_lib, F, N, H, d, fused):
+    rf = cuda_lib
+    D = H * d
+    g = torch.Generator(device=DEV).manual_seed(F * 17 + N + D)
+    if fused:
+        qkv = torch.randn(F * N, 3, D, generator=g, device=DEV).to(torch.bfloat16)
+        K, V = qkv[:, 1], qkv[:, 2]
+    else:
+        K = torch.randn(F * N, D, generator=g, device=DEV).to(torch.bfloat16)
+        V = torch.randn(F * N, D, generator=g, device=DEV).to(torch.bfloat16)
+    Kc = torch.randn(2, F, N, D, generator=g, device=DEV).to(torch.bfloat16)
+    Vc = torch.randn(2, F, N, D, generator=g, device=DEV).to(torch.bfloat16)
+    rng = np.random.default_rng(F + N)
+    mask = (rng.random(F) < 0.4).astype(np.uint8)
+    slot = rng.integers(0, 2, F).astype(np.uint8)
+    alpha = rng.random(F).astype(np.float32)
+    alpha[mask == 1] = 1.0
+    beta = (1.0 - alpha.astype(np.float64)).astype(np.float32)
+    K0, V0, Kc0, Vc0 = (x.cpu().clone() for x in (K, V, Kc, Vc))
+    act = torch.zeros(F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(torch.from_numpy(mask).to(DEV), F, N, act, skp, None, cnt)
+    rf.rf_project_kv(K, V, K.stride(0), Kc, Vc, torch.from_numpy(slot).to(DEV),
+                     torch.from_numpy(alpha).to(DEV), torch.from_numpy(beta).to(DEV), act, skp,
+                     cnt, F, N, D)
+    torch.cuda.synchronize()
+    for X, X0, Xc, Xc0 in ((K, K0, Kc, Kc0), (V, V0, Vc, Vc0)):
+        want, want_c = oracle.project_kv_cache(X0.view(F, N, D), Xc0, slot, alpha, mask)
+        got = X.cpu().double().view(F, N, D).numpy()
+        idx = np.arange(F)
+        c0 = Xc0.double().numpy()
+        sl = slot.astype(np.int64)
+        terms = (np.abs(beta.astype(np.float64))[:, None, None] * np.abs(c0[1 - sl, idx])
+                 + np.abs(alpha.astype(np.float64))[:, None, None] * np.abs(c0[sl, idx]))
+        sk = mask == 0
+        err = np.abs(got[sk] - want[sk])
+        assert (err <= 2.0 ** -8 * np.abs(terms[sk]) + 1e-30).all(), err.max()
+        np.testing.assert_array_equal(got[~sk], X0.view(F, N, D).double().numpy()[~sk])
+        # caches: active frames' other slot holds the fresh rows, everything else untouched
+        np.testing.assert_array_equal(Xc.cpu().double().numpy(), want_c)
+    if fused:
+        assert torch.equal(qkv[:, 0].cpu(), qkv[:, 0].cpu())  # Q untouched by construction
+
+
+def test_project_kv_then_attention_matches_oracle(cuda_lib):
+    """The step's keys/values of skipped frames come from the cache projection; attention
+    of the active frames over them matches the oracle computed on the projected K/V."""
+    rf = cuda_lib
+    F, N, H, d = 4, 256, 2, 128
+    D = H * d
+    g = torch.Generator(device=DEV).manual_seed(7)
+    Q, K, V = (torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
+               for _ in range(3))
+    Kc, Vc = (torch.randn(2, F, N, D, generator=g, device=DEV).to(torch.bfloat16)
+              for _ in range(2))
+    mask = np.array([1, 0, 0, 1], np.uint8)
+    slot = np.array([0, 1, 0, 1], np.uint8)
+    alpha = np.array([1.0, 0.25, 0.5, 1.0], np.float32)
+    beta = (1.0 - alpha.astype(np.float64)).astype(np.float32)
+    act = torch.zeros(F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(torch.from_numpy(mask).to(DEV), F, N, act, skp, None, cnt)
+    rf.rf_project_kv(K, V, K.stride(0), Kc, Vc, torch.from_numpy(slot).to(DEV),
+                     torch.from_numpy(alpha).to(DEV), torch.from_numpy(beta).to(DEV), act, skp,
+                     cnt, F, N, D)
+    O = torch.full_like(Q, SENTINEL)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    rf.rf_attn(O, None, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt,
+               1 / math.sqrt(d), None, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    rows = _active_rows(mask, N)
+    Oref, _ = oracle.attention(Q.cpu(), K.cpu(), V.cpu(), rows, 1 / math.sqrt(d))
+    compare(O.cpu().float()[rows].numpy(), Oref, label="attention over projected K/V")

@@ -331,3 +331,54 @@ def test_keyframes_threshold_direction():
     assert k == [0, 1, 2, 3]
     k, _ = oracle.keyframe_select(P, M=4, tau=tau0, dtau=-0.3, delta_up=1, delta_down=0)
     assert k == [0, 1, 3]
+
+
+# --------------------------------------------------------------------------
+# Rolling key/value cache (Appendix B.2)
+# --------------------------------------------------------------------------
+def _kv_case(seed, F=5, N=3, D=8):
+    rng = np.random.default_rng(seed)
+    kv = rng.standard_normal((F, N, D))
+    cache = rng.standard_normal((2, F, N, D))
+    slot = rng.integers(0, 2, F)
+    alpha = rng.random(F)
+    mask = np.array([1, 0, 1, 0, 0][:F])
+    return kv, cache, slot, alpha, mask
+
+
+def test_kv_cache_endpoints_and_store():
+    kv, cache, slot, alpha, mask = _kv_case(0)
+    alpha[:] = 0.0
+    out, c = oracle.project_kv_cache(kv, cache, slot, alpha, mask)
+    for f in range(5):
+        if mask[f]:
+            np.testing.assert_array_equal(out[f], kv[f])                  # fresh rows kept
+            np.testing.assert_array_equal(c[1 - slot[f], f], kv[f])       # shifted into cache
+            np.testing.assert_array_equal(c[slot[f], f], cache[slot[f], f])
+        else:
+            np.testing.assert_array_equal(out[f], cache[1 - slot[f], f])  # alpha 0: "before"
+            np.testing.assert_array_equal(c[:, f], cache[:, f])           # cache untouched
+    alpha[:] = 1.0
+    out, _ = oracle.project_kv_cache(kv, cache, slot, alpha, mask)
+    for f in np.flatnonzero(mask == 0):
+        np.testing.assert_array_equal(out[f], cache[slot[f], f])          # alpha 1: "after"
+
+
+def test_kv_cache_commutes_with_affine_map():
+    """Keys and values are an affine map of the hidden state (K = h W + b).  Projecting
+    cached keys equals mapping the projected hidden state: the two computation orders
+    agree for any weights (a transposed slot or a dropped (1 - alpha) breaks this)."""
+    rng = np.random.default_rng(1)
+    F, N, C, D = 4, 6, 5, 7
+    z = rng.standard_normal((2, F, N, C))
+    W = rng.standard_normal((C, D))
+    b = rng.standard_normal(D)
+    slot = np.array([0, 1, 1, 0])
+    alpha = np.array([0.3, 0.0, 0.75, 0.5])
+    mask = np.array([0, 0, 0, 1])
+    kv_fresh = rng.standard_normal((F, N, D))
+    out, _ = oracle.project_kv_cache(kv_fresh, z @ W + b, slot, alpha, mask)
+    idx = np.arange(F)
+    zp = oracle.project(z[1 - slot, idx].reshape(F, -1), z[slot, idx].reshape(F, -1), alpha)
+    want = zp.reshape(F, N, C) @ W + b
+    np.testing.assert_allclose(out[:3], want[:3], rtol=0, atol=1e-12)
