@@ -395,6 +395,27 @@ def run_bandwidth(w, dev, peaks):
                               f"A={nact}"}
     res["rf_project_kv"]["shape"] = (f"K and V bf16 [{F * w.N}][{D}] + caches [2][{F}][{w.N}]"
                                      f"[{D}], step {s}, A={A}")
+    # keyframe selection's inner products: proxies at latent width (where Algorithm 1 runs)
+    # and at the hidden-width stress shape
+    G = torch.empty(F, F, dtype=torch.float64, device=dev)
+    for label, P in (("rf_frame_gram_latent", wl.latents(w, device=dev)), ("rf_frame_gram", z2[0])):
+        times = []
+        for rep in range(13):
+            flush.fill_(rep)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            rf.rf_frame_gram(P, G)
+            b.record()
+            torch.cuda.synchronize()
+            if rep >= 3:
+                times.append(a.elapsed_time(b))
+        ms = statistics.median(times)
+        nbytes = P.numel() * 4
+        res[label] = {"GB/s": round(nbytes / (ms * 1e-3) / 1e9, 1),
+                      "frac": round(nbytes / (ms * 1e-3) / 1e9 / peaks["hbm_gbs"], 4),
+                      "peak": peaks["hbm_gbs"], "ms": round(ms, 4), "bytes": nbytes,
+                      "shape": f"F={F} proxies x E={P.shape[1]} fp32 -> [{F}][{F}] fp64"}
     del z2, ctx, v, flush, Kb, Vb, Kc, Vc
     torch.cuda.empty_cache()
     return res

@@ -253,6 +253,38 @@ rf_status rf_step(float* d_z2, const uint8_t* d_cur_slot, const float* d_v, cons
                   rf_stream_t stream);
 
 /*
+ * rf_frame_gram -- inner products of the F clean-latent proxies, the input of sequential
+ * keyframe selection (Sec. 3.1, Eq. 1; Algorithm 1 compares frames by cosine similarity).
+ *
+ *   d_P   fp32 [F][ld] proxies (frame f's E elements at d_P + f*ld), 1 <= F <= 64, ld >= E
+ *   d_G   fp64 [F][F] output, G[i][j] = sum_e P[i][e] * P[j][e]; the call zero-fills it on
+ *         `stream` first (partial sums are added with atomics, so summation order varies
+ *         between runs at the level of fp64 rounding)
+ * Per-CTA partial products are fp32 (each over at most E / #SMs / 2 elements), accumulated
+ * across CTAs in fp64.
+ */
+rf_status rf_frame_gram(const float* d_P, int F, int64_t E, int64_t ld, double* d_G,
+                        rf_stream_t stream);
+
+/*
+ * rf_keyframe_select -- Algorithm 1 (dynamic sequential keyframe selection) on the host,
+ * over a host copy of rf_frame_gram's result.
+ *
+ *   h_G        fp64 [F][F] inner products (diagonal > 0)
+ *   M          keyframe budget (>= 1); tau, dtau, delta_up, delta_down as in Algorithm 1
+ *              (the paper gives no values)
+ *   h_is_key   [F] output, 1 = keyframe; h_num_keys (nullable) output count
+ * Frame 0 is always a keyframe.  Visiting frames in order while fewer than M keyframes
+ * exist, a frame whose cosine similarity to the latest keyframe is below tau becomes one;
+ * first tau -= dtau if the gap to the latest keyframe is >= F/M + delta_up, or
+ * tau += dtau if it is <= F/M - delta_down (Algorithm 1 as printed; a negative dtau gives
+ * the adjustment direction its prose describes).
+ */
+rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double dtau,
+                             double delta_up, double delta_down, uint8_t* h_is_key,
+                             int32_t* h_num_keys);
+
+/*
  * rf_selftest_bounded_wait -- check, on the GPU, the path every device-side wait
  * of rf_attn takes when it runs out of time.  No paper passage: this is a
  * failure-handling self-test.

@@ -16,7 +16,7 @@ import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
            "rf_project", "rf_project_kv", "rf_attn", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
-           "rf_status_str",
+           "rf_frame_gram", "rf_keyframe_select", "rf_status_str",
            "rf_version", "EXPORTS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -26,7 +26,8 @@ _LIB: Optional[ctypes.CDLL] = None
 EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
            "rf_schedule_compact", "rf_project", "rf_project_kv", "rf_attn",
            "rf_attn_workspace_bytes",
-           "rf_attn_noalloc", "rf_step", "rf_selftest_bounded_wait")
+           "rf_attn_noalloc", "rf_step", "rf_frame_gram", "rf_keyframe_select",
+           "rf_selftest_bounded_wait")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
 _SIG = {
@@ -42,6 +43,9 @@ _SIG = {
                  _vp, _i64, _vp, _vp], _i32),
     "rf_attn_workspace_bytes": ([_i32], _i64),
     "rf_selftest_bounded_wait": ([_vp, _i32, _vp], _i32),
+    "rf_frame_gram": ([_vp, _i32, _i64, _i64, _vp, _vp], _i32),
+    "rf_keyframe_select": ([_vp, _i32, _i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                            ctypes.c_double, _vp, _vp], _i32),
     "rf_attn_noalloc": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
                          _f32, _vp, _vp], _i32),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
@@ -165,6 +169,24 @@ def rf_selftest_bounded_wait(status, limit_us: int, stream=None):
     """Run the device bounded-wait self-test; *status receives RF_ERR_DEVICE_TIMEOUT."""
     _check("rf_selftest_bounded_wait", load().rf_selftest_bounded_wait(
         _ptr(status), int(limit_us), _stream(stream)))
+
+
+def rf_frame_gram(P, G, stream=None):
+    """G[i][j] = <P_i, P_j> for fp32 proxies P [F, E] (row stride P.stride(0)) into fp64 G."""
+    F, E = P.shape
+    _check("rf_frame_gram", load().rf_frame_gram(_ptr(P), F, E, P.stride(0), _ptr(G),
+                                                 _stream(stream)))
+
+
+def rf_keyframe_select(G, M: int, tau: float, dtau: float, delta_up: float, delta_down: float):
+    """Algorithm 1 over a host fp64 Gram matrix; returns the keyframe mask (uint8 [F])."""
+    G = np.ascontiguousarray(np.asarray(G, dtype=np.float64))
+    F = G.shape[0]
+    is_key = np.zeros(F, np.uint8)
+    n = np.zeros(1, np.int32)
+    _check("rf_keyframe_select", load().rf_keyframe_select(
+        _ptr(G), F, M, tau, dtau, delta_up, delta_down, _ptr(is_key), _ptr(n)))
+    return is_key
 
 
 def rf_attn_workspace_bytes(d: int) -> int:

@@ -60,3 +60,39 @@ extern "C" rf_status rf_plan_build(int F, int S, const uint8_t* h_is_key, const 
   }
   return RF_OK;
 }
+
+// Algorithm 1 (dynamic sequential keyframe selection) over the frames' inner products.
+// Frame 0 is the first keyframe.  Frames are visited in order; while fewer than M keyframes
+// exist, a frame whose cosine similarity to the latest keyframe is below tau becomes a
+// keyframe, after tau is moved by -dtau if the gap to the latest keyframe is at least
+// F/M + delta_up, or by +dtau if it is at most F/M - delta_down (Algorithm 1 as printed).
+extern "C" rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double dtau,
+                                        double delta_up, double delta_down, uint8_t* h_is_key,
+                                        int32_t* h_num_keys) {
+  if (!h_G || !h_is_key || F < 1 || M < 1) return RF_ERR_INVALID_ARG;
+  for (int f = 0; f < F; ++f) {
+    h_is_key[f] = 0;
+    if (!(h_G[static_cast<size_t>(f) * F + f] > 0.0)) return RF_ERR_INVALID_ARG;  // zero frame
+  }
+  h_is_key[0] = 1;
+  int keys = 1, last = 0;
+  const double L_avg = static_cast<double>(F) / M;
+  for (int i = 1; i < F; ++i) {
+    if (keys >= M) break;
+    const double gii = h_G[static_cast<size_t>(i) * F + i];
+    const double gll = h_G[static_cast<size_t>(last) * F + last];
+    const double sim = h_G[static_cast<size_t>(i) * F + last] / (std::sqrt(gii) * std::sqrt(gll));
+    if (sim < tau) {
+      const int gap = i - last;
+      if (gap >= L_avg + delta_up)
+        tau -= dtau;
+      else if (gap <= L_avg - delta_down)
+        tau += dtau;
+      h_is_key[i] = 1;
+      ++keys;
+      last = i;
+    }
+  }
+  if (h_num_keys) *h_num_keys = keys;
+  return RF_OK;
+}

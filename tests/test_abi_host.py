@@ -106,3 +106,34 @@ def test_device_calls_reject_bad_args_on_host(rf):
     args[14], args[15] = P, -1
     assert lib.rf_attn(*args) == 1                                   # negative workspace size
     assert lib.rf_attn_workspace_bytes(96) == -1
+
+
+def _scene_proxies(F=21, E=960, starts=(0, 4, 9, 13, 17), noise=0.3, seed=0):
+    rng = np.random.default_rng(seed)
+    base = rng.standard_normal((len(starts), E))
+    scene = np.searchsorted(np.array(starts), np.arange(F), side="right") - 1
+    return base[scene] + noise * rng.standard_normal((F, E))
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_keyframe_select_host_matches_oracle(rf, seed):
+    """Algorithm 1 on the host over inner products equals the oracle working on the
+    proxies directly, over random thresholds, budgets and tolerances."""
+    rng = np.random.default_rng(100 + seed)
+    P = _scene_proxies(seed=seed, noise=float(rng.uniform(0.1, 1.5)))
+    G = P @ P.T
+    for _ in range(20):
+        M = int(rng.integers(1, 22))
+        tau, dtau = float(rng.uniform(-0.2, 1.0)), float(rng.uniform(-0.3, 0.3))
+        up, down = float(rng.uniform(0, 4)), float(rng.uniform(0, 4))
+        got = rf.rf_keyframe_select(G, M, tau, dtau, up, down)
+        keys, _ = oracle.keyframe_select(P, M, tau, dtau, up, down)
+        assert np.flatnonzero(got).tolist() == keys, (M, tau, dtau, up, down)
+
+
+def test_keyframe_select_scene_starts(rf):
+    P = _scene_proxies()
+    got = rf.rf_keyframe_select(P @ P.T, 8, 0.5, 0.0, 1.0, 1.0)
+    assert np.flatnonzero(got).tolist() == [0, 4, 9, 13, 17]
+    with pytest.raises(rf.RFError):
+        rf.rf_keyframe_select(np.zeros((3, 3)), 2, 0.5, 0.0, 1, 1)   # zero-norm frames

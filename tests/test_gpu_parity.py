@@ -473,3 +473,44 @@ def test_project_kv_then_attention_matches_oracle(cuda_lib):
     rows = _active_rows(mask, N)
     Oref, _ = oracle.attention(Q.cpu(), K.cpu(), V.cpu(), rows, 1 / math.sqrt(d))
     compare(O.cpu().float()[rows].numpy(), Oref, label="attention over projected K/V")
+
+
+# ---------------------------------------------------------------------------
+# Keyframe selection: inner products on the device, Algorithm 1 on the host
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("F,E,ld", [(21, 3600 * 16, 3600 * 16), (33, 1000, 1003), (1, 37, 37),
+                                    (64, 4096, 4096), (13, 1560 * 16 * 12, 1560 * 16 * 12),
+                                    (40, 777, 780), (17, 129, 132)])
+def test_frame_gram_matches_fp64_matmul(cuda_lib, F, E, ld):
+    rf = cuda_lib
+    g = torch.Generator(device=DEV).manual_seed(F + E)
+    Pfull = torch.randn(F, ld, generator=g, device=DEV)
+    P = Pfull[:, :E]
+    G = torch.full((F, F), 7.0, dtype=torch.float64, device=DEV)
+    rf.rf_frame_gram(P, G)
+    torch.cuda.synchronize()
+    ref = P.double().cpu().numpy() @ P.double().cpu().numpy().T
+    scale = np.sqrt(np.outer(np.diag(ref), np.diag(ref)))
+    err = np.abs(G.cpu().numpy() - ref) / scale
+    assert err.max() < 1e-5, err.max()
+
+
+def test_keyframes_from_device_gram_match_oracle(cuda_lib):
+    """Scene-structured proxies (5 scenes over 21 frames of 3600 tokens x 16 channels):
+    the keyframes are the scene starts, as the oracle's Algorithm 1 finds them."""
+    rf = cuda_lib
+    F, E, starts = 21, 3600 * 16, (0, 4, 9, 13, 17)
+    rng = np.random.default_rng(3)
+    base = rng.standard_normal((len(starts), E))
+    scene = np.searchsorted(np.array(starts), np.arange(F), side="right") - 1
+    P = base[scene] + 0.3 * rng.standard_normal((F, E))
+    Pd = torch.from_numpy(P.astype(np.float32)).to(DEV)
+    G = torch.empty(F, F, dtype=torch.float64, device=DEV)
+    rf.rf_frame_gram(Pd, G)
+    torch.cuda.synchronize()
+    for M, tau, dtau in ((8, 0.5, 0.0), (4, 0.5, 0.1), (6, 0.95, -0.2)):
+        got = np.flatnonzero(rf.rf_keyframe_select(G.cpu().numpy(), M, tau, dtau, 1.0, 1.0))
+        want, _ = oracle.keyframe_select(P.astype(np.float32), M, tau, dtau, 1.0, 1.0)
+        assert got.tolist() == want, (M, tau, dtau)
+    assert np.flatnonzero(rf.rf_keyframe_select(G.cpu().numpy(), 8, 0.5, 0.0, 1, 1)).tolist() == \
+        list(starts)
