@@ -253,24 +253,25 @@ drain:
 // ---------------------------------------------------------------------------------------
 // MMA issuer (one thread).
 // ---------------------------------------------------------------------------------------
+// Descriptors are built once per buffer; a K step only adds its byte offset / 16 to the start
+// address field (bits 0-13), which cannot carry: every shared address is below 256 KB.  (The
+// single issuing thread is on the critical path: rebuilding descriptors per MMA cost ~2-4%.)
 template <int D>
-__device__ __forceinline__ void mma_qk(uint32_t tS, uint32_t sQ, uint32_t sK) {
+__device__ __forceinline__ void mma_qk(uint32_t tS, uint64_t dQ, uint64_t dK) {
   constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, 0, 0);
 #pragma unroll
   for (int k = 0; k < D / 16; ++k) {
-    const uint32_t off = (k >> 2) * (BM * 128) + (k & 3) * 32;
-    tc_mma_ss(tS, smem_desc_sw128(sQ + off, 16, 1024), smem_desc_sw128(sK + off, 16, 1024), idesc,
-              k > 0);
+    const uint64_t off = ((k >> 2) * (BM * 128) + (k & 3) * 32) >> 4;
+    tc_mma_ss(tS, dQ + off, dK + off, idesc, k > 0);
   }
 }
 
 template <int D>
-__device__ __forceinline__ void mma_pv(uint32_t tO, uint32_t tP, uint32_t sV, uint32_t acc) {
+__device__ __forceinline__ void mma_pv(uint32_t tO, uint32_t tP, uint64_t dV, uint32_t acc) {
   constexpr uint32_t idesc = idesc_bf16_f32(BM, D, 0, 1);
 #pragma unroll
   for (int k = 0; k < BN / 16; ++k)
-    tc_mma_ts(tO, tP + k * 8, smem_desc_sw128(sV + k * 2048, BN * 128, 1024), idesc,
-              (acc | k) != 0);
+    tc_mma_ts(tO, tP + k * 8, dV + ((k * 2048) >> 4), idesc, (acc | k) != 0);
 }
 
 template <int D>
@@ -281,7 +282,11 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
   auto bar = [&](int i) { return bar0 + 8u * i; };
   const uint32_t tS[2] = {tmem, tmem + 128};
   const uint32_t tO[2] = {tmem + 256, tmem + 384};
-  const uint32_t sQ[2] = {sQ0, sQ0 + C::kTileBytes};
+  const uint64_t dQ[2] = {smem_desc_sw128(sQ0, 16, 1024),
+                          smem_desc_sw128(sQ0 + C::kTileBytes, 16, 1024)};
+  // K operand: K-major; V operand: MN-major with the two 64-column halves 16 KB apart
+  auto dK = [&](int s) { return smem_desc_sw128(sKV0 + s * C::kTileBytes, 16, 1024); };
+  auto dV = [&](int s) { return smem_desc_sw128(sKV0 + s * C::kTileBytes, BN * 128, 1024); };
   int q_cnt[2] = {0, 0};
   int p_cnt[2] = {0, 0};
   int it = 0;
@@ -311,40 +316,40 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     tc_fence_after();
     int sK, sV;
     if (!next_slot(sK)) goto fail;
-    mma_qk<D>(tS[0], sQ[0], sKV0 + sK * C::kTileBytes);
+    mma_qk<D>(tS[0], dQ[0], dK(sK));
     tc_commit(bar(C::kBarSFull + 0));
     if (hasB) {
-      mma_qk<D>(tS[1], sQ[1], sKV0 + sK * C::kTileBytes);
+      mma_qk<D>(tS[1], dQ[1], dK(sK));
       tc_commit(bar(C::kBarSFull + 1));
     }
     tc_commit(bar(C::kBarKVEmpty + sK));
     if (!next_slot(sV)) goto fail;
     if (!wait_p(0)) goto fail;
-    mma_pv<D>(tO[0], tS[0], sKV0 + sV * C::kTileBytes, 0);
+    mma_pv<D>(tO[0], tS[0], dV(sV), 0);
 #pragma unroll 1
     for (int j = 0; j + 1 < nj; ++j) {
       if (!next_slot(sK)) goto fail;
-      mma_qk<D>(tS[0], sQ[0], sKV0 + sK * C::kTileBytes);
+      mma_qk<D>(tS[0], dQ[0], dK(sK));
       tc_commit(bar(C::kBarSFull + 0));
       if (hasB) {
         if (!wait_p(1)) goto fail;
-        mma_pv<D>(tO[1], tS[1], sKV0 + sV * C::kTileBytes, j > 0);
+        mma_pv<D>(tO[1], tS[1], dV(sV), j > 0);
       }
       tc_commit(bar(C::kBarKVEmpty + sV));
       if (hasB) {
-        mma_qk<D>(tS[1], sQ[1], sKV0 + sK * C::kTileBytes);
+        mma_qk<D>(tS[1], dQ[1], dK(sK));
         tc_commit(bar(C::kBarSFull + 1));
       }
       tc_commit(bar(C::kBarKVEmpty + sK));
       if (!next_slot(sV)) goto fail;
       if (!wait_p(0)) goto fail;
-      mma_pv<D>(tO[0], tS[0], sKV0 + sV * C::kTileBytes, 1);
+      mma_pv<D>(tO[0], tS[0], dV(sV), 1);
     }
     tc_commit(bar(C::kBarODone + 0));
     tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       if (!wait_p(1)) goto fail;
-      mma_pv<D>(tO[1], tS[1], sKV0 + sV * C::kTileBytes, nj > 1);
+      mma_pv<D>(tO[1], tS[1], dV(sV), nj > 1);
       tc_commit(bar(C::kBarODone + 1));
       tc_commit(bar(C::kBarQEmpty + 1));
     }
