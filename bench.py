@@ -230,6 +230,24 @@ def run_gpu(args):
     per_launch_flops = attn_flops_total / len(ev)
     # all-frames-active comparison, same number of steps
     ms_all, _ = timed(core_all, K_steps, min(W_steps, 3))
+    # the same trajectory replayed from one CUDA graph (launch overhead removed)
+    graph_ms = None
+    try:
+        g = core.capture_trajectory(vel, O, Q, K, V, w.softmax_scale)
+        reps = max(1, K_steps // S)
+        g.replay()
+        barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+        barrier()
+        graph_ms = a.elapsed_time(b) / (reps * S)
+        del g
+    except RuntimeError as e:  # report, never hide: the eager numbers above stand
+        graph_ms = f"capture failed: {e}"
 
     # end to end through the public API with host buffers
     e2e = run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist, world)
@@ -259,6 +277,7 @@ def run_gpu(args):
         },
         "step_core_ms": round(ms / K_steps, 5),
         "step_core_ms_all_active": round(ms_all / K_steps, 5),
+        "step_core_ms_cuda_graph": round(graph_ms, 5) if isinstance(graph_ms, float) else graph_ms,
         "speedup_vs_all_active": round(ms_all / ms, 4),
         "ideal_speedup_vs_all_active": round(K_steps * flops_all /
                                              sum(flops_step[k % S] for k in range(K_steps)), 4),

@@ -97,6 +97,23 @@ class StepCore:
         self.attn(O, Q, K, V, scale, lse, stream)
         self.step(s, v, stream)
 
+    def capture_trajectory(self, vels, O, Q, K, V, scale: float, steps=None):
+        """Record steps 0..S-1 (4 launches each) into one CUDA graph and return it.
+
+        Nothing in the step core synchronises the host (counts stay on the device), so the
+        whole trajectory replays with one launch.  Every call is made once eagerly first, so
+        one-time host set-up (kernel attributes, entry points) happens outside the capture.
+        Replaying advances the latent store exactly as the eager steps would.
+        """
+        S = self.plan.mask.shape[0] if steps is None else steps
+        self.run(0, vels[0], O, Q, K, V, scale)  # warm-up outside the capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for s in range(S):
+                self.run(s, vels[s], O, Q, K, V, scale)
+        return g
+
 
 class HostPipeline:
     """Step-core steps fed from pinned host memory, with the copies hidden behind compute.

@@ -514,3 +514,37 @@ def test_keyframes_from_device_gram_match_oracle(cuda_lib):
         assert got.tolist() == want, (M, tau, dtau)
     assert np.flatnonzero(rf.rf_keyframe_select(G.cpu().numpy(), 8, 0.5, 0.0, 1, 1)).tolist() == \
         list(starts)
+
+
+@pytest.mark.parametrize("name", ["tiny", "small"])
+def test_graph_replay_matches_eager(cuda_lib, name):
+    """A whole trajectory captured in one CUDA graph and replayed gives the eager results."""
+    from paper_2606_06309_gb300.stepcore import StepCore, upload_plan
+    w = wl.get(name)
+    E = w.N * w.C
+    Q, K, V = wl.qkv(w, device=DEV)
+    vels = [wl.velocity(w, s, device=DEV) for s in range(w.S)]
+    z0 = wl.latents(w, device=DEV)
+
+    def fresh():
+        plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, DEV)
+        c = StepCore(w.F, w.N, E, w.H, w.d, plan, DEV)
+        c.set_state(z0)
+        return c
+
+    eager = fresh()
+    O1 = torch.zeros_like(Q)
+    for s in range(w.S):
+        eager.run(s, vels[s], O1, Q, K, V, w.softmax_scale)
+    torch.cuda.synchronize()
+
+    cg = fresh()
+    O2 = torch.zeros_like(Q)
+    g = cg.capture_trajectory(vels, O2, Q, K, V, w.softmax_scale)  # runs step 0 once eagerly
+    cg.set_state(z0)
+    O2.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(cg.z2, eager.z2)
+    assert torch.equal(O1, O2)
+    assert cg.status.item() == 0
