@@ -259,6 +259,7 @@ def run_gpu(args):
         traffic = ATTN_TRAFFIC["bytes_per_launch"]
     bw = run_bandwidth(w, dev, peaks) if not args.no_bandwidth else None
     sweep = run_sweep(w, dev, Q, K, V, O, vel, max(3, min(K_steps, 10))) if w.sweep else None
+    block = run_block_mask(w, dev, Q, K, V, O, plan, core) if not args.no_bandwidth else None
     status = int(core.status.item()) | int(core_all.status.item())
 
     out = {
@@ -293,6 +294,7 @@ def run_gpu(args):
         },
         "bandwidth_kernels": bw,
         "active_fraction_sweep": sweep,
+        "combined_block_mask": block,
         "e2e": e2e,
         "gpu_launches": 4 * K_steps,
         "clocks": clocks,
@@ -438,6 +440,57 @@ def run_bandwidth(w, dev, peaks):
     del z2, ctx, v, flush, Kb, Vb, Kc, Vc
     torch.cuda.empty_cache()
     return res
+
+
+def run_block_mask(w, dev, Q, K, V, O, plan, core, reps=10):
+    """Frame mask x token block mask (the paper's combined mask): attention of a step with a
+    synthetic banded block mask (query block qb may attend to key blocks |qb - kb| <= band,
+    about a quarter of all blocks) next to the same step unmasked.  FLOPs count allowed
+    (query row, key) pairs only."""
+    import numpy as np
+    import torch
+    import paper_2606_06309_gb300 as rf
+    nb = (w.S_tok + 127) // 128
+    band = max(1, nb // 8)
+    qb, kb = np.meshgrid(np.arange(nb), np.arange(nb), indexing="ij")
+    bm = np.broadcast_to((np.abs(qb - kb) <= band).astype(np.uint8), (w.H, nb, nb)).copy()
+    bm_d = torch.from_numpy(bm).to(dev)
+    out = {"band_blocks": band, "density": round(float(bm[0].mean()), 4), "steps": {}}
+    key_len = np.array([min(128, w.S_tok - 128 * k) for k in range(nb)])
+    for s in (0, 1) if w.S > 1 else (0,):
+        core.compact(s)
+        mask = plan.host["mask"][s]
+        rows = np.array([f * w.N + p for f in range(w.F) if mask[f] for p in range(w.N)])
+        allowed_keys = (bm[0][rows // 128] * key_len[None, :]).sum()
+        flops = 4 * int(allowed_keys) * w.d * w.H
+        res = {}
+        for label, fn in (
+                ("unmasked", lambda: rf.rf_attn(O, None, Q, K, V, Q.stride(0), O.stride(0), w.F,
+                                                w.N, w.H, w.d, core.active, core.counts,
+                                                w.softmax_scale, core.workspace, core.status)),
+                ("block_masked", lambda: rf.rf_attn_block_masked(
+                    O, None, Q, K, V, Q.stride(0), O.stride(0), w.F, w.N, w.H, w.d, core.active,
+                    core.counts, w.softmax_scale, bm_d, core.workspace, core.status))):
+            for _ in range(3):
+                fn()
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(reps):
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                fn()
+                b.record()
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(b))
+            res[label] = statistics.median(ts)
+        out["steps"][str(s)] = {
+            "active_frames": int(mask.sum()), "unmasked_ms": round(res["unmasked"], 4),
+            "block_masked_ms": round(res["block_masked"], 4),
+            "speedup": round(res["unmasked"] / res["block_masked"], 3),
+            "ideal_speedup": round(4 * len(rows) * w.S_tok * w.d * w.H / flops, 3),
+            "masked_tflops": round(flops / (res["block_masked"] * 1e-3) / 1e12, 1)}
+    return out
 
 
 def run_sweep(w, dev, Q, K, V, O, vel, steps):

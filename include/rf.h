@@ -196,6 +196,26 @@ rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K, con
                   rf_stream_t stream);
 
 /*
+ * rf_attn_block_masked -- rf_attn under the combined mask of Appendix D:
+ * M_combined = M_Rhyme (element-wise) M_SAP.  M_Rhyme, the frame mask, is the active list
+ * (only active frames' queries are computed, as in rf_attn); M_SAP is a token-level block
+ * mask:
+ *   d_block_mask  uint8 [H][nb][nb], nb = ceil(F*N / 128): entry [h][qb][kb] nonzero lets
+ *                 query tokens 128*qb .. 128*qb+127 attend to key tokens 128*kb .. 128*kb+127
+ *                 for head h (blocks over the token index t = f*N + p of the whole sequence)
+ * Keys a row may not attend to are excluded from its softmax; key blocks no query row of a
+ * work item may attend to are not loaded or multiplied at all.  A row that may attend to
+ * no key gets O = 0 and LSE = -inf.  All other arguments, requirements and results are
+ * those of rf_attn.  Returns RF_ERR_INVALID_ARG for a null mask.
+ */
+rf_status rf_attn_block_masked(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
+                               const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride,
+                               int F, int N, int H, int d, const int32_t* d_active,
+                               const int32_t* d_counts, float softmax_scale,
+                               const uint8_t* d_block_mask, void* d_workspace,
+                               int64_t workspace_bytes, int32_t* d_status, rf_stream_t stream);
+
+/*
  * rf_attn_workspace_bytes -- bytes of split-KV workspace rf_attn can use on the
  * current device for head dim d (independent of the problem size: counters plus
  * one partial result tile per SM).  Returns -1 for an unsupported d or when the

@@ -10,5 +10,5 @@ Everything is plain, slow fp64 numpy (pure Python loops for the schedule).
 """
 from .rf_oracle import (  # noqa: F401
     sigmas, schedule, active_set_alg2, compact, project, attention, euler,
-    sampler, flops_attn, keyframe_select, project_kv_cache, to_f64,
+    sampler, flops_attn, keyframe_select, project_kv_cache, attention_block_masked, to_f64,
 )

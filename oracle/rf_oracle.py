@@ -18,6 +18,9 @@ Citations name the paper's sections, equations and algorithms:
                        attention in fp64, brute force over every key.
 * euler()           -- the heterogeneous update of Algorithm 2 / Sec. 3.2.3 as a
                        rectified-flow Euler step z <- z + (sigma_to - sigma_from) v.
+* attention_block_masked() -- Appendix D, Eq. (combined mask): the frame-level mask of the
+                       method times a token-level block mask; active queries attend only
+                       to the key blocks their query block allows.
 * project_kv_cache() -- Appendix B.2, per-layer rolling cache: skipped frames'
                        keys/values projected with Eq. 3 from the two cached states,
                        active frames' fresh keys/values shifted into the cache.
@@ -35,7 +38,8 @@ from typing import Dict, Optional, Sequence
 import numpy as np
 
 __all__ = ["sigmas", "schedule", "active_set_alg2", "compact", "project", "attention",
-           "euler", "sampler", "flops_attn", "keyframe_select", "project_kv_cache", "to_f64"]
+           "euler", "sampler", "flops_attn", "keyframe_select", "project_kv_cache",
+           "attention_block_masked", "to_f64"]
 
 
 def to_f64(x) -> np.ndarray:
@@ -212,6 +216,38 @@ def project_kv_cache(KV, cache, cur_slot, alpha, mask):
             a = float(alpha[f])
             kv[f] = (1.0 - a) * c[1 - cur, f] + a * c[cur, f]
     return kv, c
+
+
+def attention_block_masked(Q, K, V, rows, scale, block_mask, block: int = 128,
+                           heads: Optional[Sequence[int]] = None):
+    """Attention under M_combined = M_Rhyme (element-wise) M_SAP.
+
+    M_Rhyme is the step's frame mask: only the query tokens `rows` (of active frames) are
+    computed.  M_SAP is a token-level block mask, block_mask[h][qb][kb] (nonzero = allowed)
+    over blocks of `block` consecutive tokens: query token i may attend to key token j only
+    when block_mask[h][i // block][j // block] is nonzero.  Scores of excluded keys are
+    removed from the softmax.  A row with no allowed key has O = 0 and LSE = -inf.
+    """
+    Kf, Vf, Qf = to_f64(K), to_f64(V), to_f64(Q)
+    M = np.asarray(block_mask)
+    rows = np.asarray(rows, dtype=np.int64)
+    H, S_tok, d = Kf.shape[1], Kf.shape[0], Kf.shape[2]
+    heads = list(range(H)) if heads is None else list(heads)
+    kb = np.arange(S_tok) // block
+    O = np.zeros((len(rows), len(heads), d), dtype=np.float64)
+    L = np.full((len(heads), len(rows)), -np.inf, dtype=np.float64)
+    for hi, h in enumerate(heads):
+        for ri, i in enumerate(rows):
+            allowed = M[h, i // block, kb] != 0
+            if not allowed.any():
+                continue
+            s = scale * (Kf[allowed, h, :] @ Qf[i, h, :])
+            m = s.max()
+            e = np.exp(s - m)
+            l = e.sum()
+            O[ri, hi] = (e @ Vf[allowed, h, :]) / l
+            L[hi, ri] = m + np.log(l)
+    return O, L
 
 
 def euler(z, v, dt) -> np.ndarray:

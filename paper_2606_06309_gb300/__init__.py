@@ -15,7 +15,7 @@ from typing import Optional
 import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_project_kv", "rf_attn", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
+           "rf_project", "rf_project_kv", "rf_attn", "rf_attn_block_masked", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
            "rf_frame_gram", "rf_keyframe_select", "rf_status_str",
            "rf_version", "EXPORTS"]
 
@@ -25,7 +25,7 @@ _LIB: Optional[ctypes.CDLL] = None
 # Every symbol include/rf.h declares.
 EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
            "rf_schedule_compact", "rf_project", "rf_project_kv", "rf_attn",
-           "rf_attn_workspace_bytes",
+           "rf_attn_block_masked", "rf_attn_workspace_bytes",
            "rf_attn_noalloc", "rf_step", "rf_frame_gram", "rf_keyframe_select",
            "rf_selftest_bounded_wait")
 
@@ -42,6 +42,8 @@ _SIG = {
     "rf_attn": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp, _f32,
                  _vp, _i64, _vp, _vp], _i32),
     "rf_attn_workspace_bytes": ([_i32], _i64),
+    "rf_attn_block_masked": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp,
+                              _vp, _f32, _vp, _vp, _i64, _vp, _vp], _i32),
     "rf_selftest_bounded_wait": ([_vp, _i32, _vp], _i32),
     "rf_frame_gram": ([_vp, _i32, _i64, _i64, _vp, _vp], _i32),
     "rf_keyframe_select": ([_vp, _i32, _i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
@@ -154,6 +156,17 @@ def rf_attn(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: 
         _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
         _ptr(active), _ptr(counts), float(softmax_scale), _ptr(workspace), ws_bytes,
         _ptr(status), _stream(stream)))
+
+
+def rf_attn_block_masked(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int,
+                         N: int, H: int, d: int, active, counts, softmax_scale: float, block_mask,
+                         workspace=None, status=None, stream=None):
+    """rf_attn under the frame mask x token block mask (block_mask uint8 [H, nb, nb])."""
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check("rf_attn_block_masked", load().rf_attn_block_masked(
+        _ptr(O), _ptr(lse), _ptr(Q), _ptr(K), _ptr(V), qkv_row_stride, o_row_stride, F, N, H, d,
+        _ptr(active), _ptr(counts), float(softmax_scale), _ptr(block_mask), _ptr(workspace),
+        ws_bytes, _ptr(status), _stream(stream)))
 
 
 def rf_attn_noalloc(O, lse, Q, K, V, qkv_row_stride: int, o_row_stride: int, F: int, N: int,

@@ -93,6 +93,7 @@ struct AttnParams {
   int32_t* status;
   int* ws_count;   // [kMaxGrid] merge counters (zero between launches), or null: no split
   float* ws_part;  // [kMaxGrid][2][BM][D+4] partial rows
+  const uint8_t* block_mask;  // [H][nkv][nkv] token block mask (128-token blocks), or null
   int64_t o_row_stride;
   int F, N, Np, H, S_tok, nkv;
   float scale_log2;
@@ -164,6 +165,65 @@ __device__ __forceinline__ Unit get_unit(const Sched& s, const AttnParams& p, in
   return u;
 }
 
+// Token block mask (combined frame x token mask).  The valid query rows of a unit's tile pair
+// form runs of consecutive tokens (one per active frame they touch), so the query blocks they
+// cover are a few ranges, non-decreasing along the rows; overlapping or adjacent ranges are
+// merged and, past kMaxQRanges, the last range is extended (a superset only costs skipped
+// work, never correctness: every row still applies its own mask).
+constexpr int kMaxQRanges = 6;
+struct QRanges {
+  int n;
+  int lo[kMaxQRanges], hi[kMaxQRanges];
+  const uint8_t* mh;  // this head's [nkv][nkv] mask
+};
+
+__device__ __forceinline__ QRanges unit_qranges(const AttnParams& p, const Sched& sc,
+                                                const Unit& u) {
+  QRanges q;
+  q.n = 0;
+  q.mh = p.block_mask + static_cast<int64_t>(u.h) * p.nkv * p.nkv;
+  const int r0 = u.pr * 2 * BM;
+  const int r1 = min(r0 + 2 * BM, sc.R);
+  for (int r = r0; r < r1;) {
+    const int a = r / p.Np;
+    const int seg_end = min(r1, (a + 1) * p.Np);
+    const int p_lo = r - a * p.Np, p_hi = min(seg_end - a * p.Np, p.N) - 1;
+    if (p_lo <= p_hi) {
+      const int t0 = p.active[a] * p.N;
+      const int lo = (t0 + p_lo) / BN, hi = (t0 + p_hi) / BN;
+      if (q.n > 0 && lo <= q.hi[q.n - 1] + 1) {
+        q.hi[q.n - 1] = max(q.hi[q.n - 1], hi);
+      } else if (q.n < kMaxQRanges) {
+        q.lo[q.n] = lo;
+        q.hi[q.n] = hi;
+        ++q.n;
+      } else {
+        q.hi[q.n - 1] = max(q.hi[q.n - 1], hi);
+      }
+    }
+    r = seg_end;
+  }
+  return q;
+}
+
+// May any query block of the unit attend to key block j?
+__device__ __forceinline__ bool unit_allows(const AttnParams& p, const QRanges& q, int j) {
+  for (int i = 0; i < q.n; ++i)
+    for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb)
+      if (q.mh[static_cast<int64_t>(qb) * p.nkv + j]) return true;
+  return false;
+}
+
+// First allowed KV tile at or after j (u.j1 if none).
+template <bool MASKED>
+__device__ __forceinline__ int next_tile(const AttnParams& p, const QRanges& q, const Unit& u,
+                                         int j) {
+  if constexpr (MASKED) {
+    while (j < u.j1 && !unit_allows(p, q, j)) ++j;
+  }
+  return j;
+}
+
 __device__ __forceinline__ void flag_error(const AttnParams& p, int where) {
   if (p.status) atomicOr(p.status, RF_ERR_DEVICE_TIMEOUT | (1 << (8 + where)));
 }
@@ -188,7 +248,7 @@ __device__ __forceinline__ bool group_sync(uint32_t bar, int& cnt, volatile int*
 // ---------------------------------------------------------------------------------------
 // TMA producer (one thread).
 // ---------------------------------------------------------------------------------------
-template <int D>
+template <int D, bool MASKED>
 __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorMap* tmK,
                                          const CUtensorMap* tmV, const AttnParams& p,
                                          const Sched& sc, uint32_t sQ0, uint32_t sKV0,
@@ -199,6 +259,8 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
   int it = 0;
   for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
     const Unit u = get_unit(sc, p, w);
+    QRanges qr{};
+    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
     for (int X = 0; X < 2; ++X) {
       const int t = 2 * u.pr + X;
       if (t >= sc.tiles) break;
@@ -224,7 +286,8 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
       ++q_cnt[X];
     }
 #pragma unroll 1
-    for (int j = u.j0; j < u.j1; ++j) {
+    for (int j = next_tile<MASKED>(p, qr, u, u.j0); j < u.j1;
+         j = next_tile<MASKED>(p, qr, u, j + 1)) {
 #pragma unroll
       for (int kv = 0; kv < 2; ++kv) {
         const int s = it % C::kSlots, n = it / C::kSlots;
@@ -274,7 +337,7 @@ __device__ __forceinline__ void mma_pv(uint32_t tO, uint32_t tP, uint64_t dV, ui
     tc_mma_ts(tO, tP + k * 8, dV + ((k * 2048) >> 4), idesc, (acc | k) != 0);
 }
 
-template <int D>
+template <int D, bool MASKED>
 __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc, uint32_t tmem,
                                            uint32_t sQ0, uint32_t sKV0, uint32_t bar0,
                                            volatile int* abort) {
@@ -306,7 +369,10 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
   for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
     const Unit u = get_unit(sc, p, w);
     const bool hasB = 2 * u.pr + 1 < sc.tiles;
-    const int nj = u.j1 - u.j0;
+    // KV tiles of the unit: all of [j0, j1), or (MASKED) the allowed ones, walked in order
+    QRanges qr{};
+    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
+    int jc = next_tile<MASKED>(p, qr, u, u.j0);
     if (!mbar_wait(bar(C::kBarQFull + 0), q_cnt[0] & 1, abort, kWaitLimitNs)) goto fail;
     ++q_cnt[0];
     if (hasB) {
@@ -314,6 +380,14 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       ++q_cnt[1];
     }
     tc_fence_after();
+    if (MASKED && jc >= u.j1) {
+      // no allowed key block: release the queries.  No output barrier is committed: the
+      // softmax warps see the same empty tile list and write their result without waiting
+      // (a commit here could run two phases ahead of them).
+      tc_commit(bar(C::kBarQEmpty + 0));
+      if (hasB) tc_commit(bar(C::kBarQEmpty + 1));
+      continue;
+    }
     int sK, sV;
     if (!next_slot(sK)) goto fail;
     mma_qk<D>(tS[0], dQ[0], dK(sK));
@@ -326,8 +400,16 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     if (!next_slot(sV)) goto fail;
     if (!wait_p(0)) goto fail;
     mma_pv<D>(tO[0], tS[0], dV(sV), 0);
+    int nj = 1;  // tiles issued so far
 #pragma unroll 1
-    for (int j = 0; j + 1 < nj; ++j) {
+    for (int j = 0;; ++j) {
+      if constexpr (MASKED) {
+        jc = next_tile<MASKED>(p, qr, u, jc + 1);
+        if (jc >= u.j1) break;
+      } else {
+        if (j + 1 >= u.j1 - u.j0) break;
+      }
+      ++nj;
       if (!next_slot(sK)) goto fail;
       mma_qk<D>(tS[0], dQ[0], dK(sK));
       tc_commit(bar(C::kBarSFull + 0));
@@ -381,7 +463,7 @@ __device__ __forceinline__ void store_row_bf16(uint16_t* orow, const float* o, f
   }
 }
 
-template <int D>
+template <int D, bool MASKED>
 __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& sc, int X,
                                               uint32_t tmem, uint32_t bar0, volatile int* abort,
                                               volatile int* merge_flag) {
@@ -399,9 +481,26 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
     const Unit u = get_unit(sc, p, w);
     const int t = 2 * u.pr + X;
     if (t >= sc.tiles) continue;
+    QRanges qr{};
+    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
+    const bool empty_unit = MASKED && next_tile<MASKED>(p, qr, u, u.j0) >= u.j1;
     float m = -INFINITY, l = 0.f;
+    // this row's query block (MASKED): rows past the active list or in frame padding are
+    // never stored and need no mask
+    const uint8_t* mrow = nullptr;
+    if constexpr (MASKED) {
+      const int r = t * BM + row;
+      if (r < sc.R) {
+        const int a = r / p.Np, pp = r - a * p.Np;
+        if (pp < p.N) {
+          const int qb = (p.active[a] * p.N + pp) / BN;
+          mrow = p.block_mask + (static_cast<int64_t>(u.h) * p.nkv + qb) * p.nkv;
+        }
+      }
+    }
 #pragma unroll 1
-    for (int j = u.j0; j < u.j1; ++j) {
+    for (int j = next_tile<MASKED>(p, qr, u, u.j0); j < u.j1;
+         j = next_tile<MASKED>(p, qr, u, j + 1)) {
       // the result is made warp-uniform: tcgen05.ld/st below are warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(bar(C::kBarSFull + X), s_cnt & 1, abort,
                                             kWaitLimitNs))) {
@@ -421,6 +520,12 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         for (int c = 0; c < BN; ++c)
           if (c >= valid) sf[c] = -INFINITY;
       }
+      if constexpr (MASKED) {
+        if (mrow != nullptr && mrow[j] == 0) {
+#pragma unroll
+          for (int c = 0; c < BN; ++c) sf[c] = -INFINITY;
+        }
+      }
       // row max: 8 independent chains of three-input maxima (a single 128-long chain of
       // two-input maxima is pure latency on the path from QK^T to PV)
       float mx8[8];
@@ -437,13 +542,17 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       const bool rescale = __any_sync(0xffffffffu, need);
       float fac = 1.f;
       if (rescale) {
-        fac = ex2_approx(m - m_new);
+        // (MASKED) a row that has seen only excluded keys has m = m_new = -inf while another
+        // row of its warp asked for the rescale: factor 1, not 2^(-inf + inf)
+        fac = (MASKED && m == m_new) ? 1.f : ex2_approx(m - m_new);
         l *= fac;
         m = m_new;
       }
       // p = 2^(s*scale*log2(e) - m) with packed fp32 pairs for the scale/subtract and the
       // row sum (8 independent sum chains in 4 packed accumulators)
-      const uint64_t sl2x2 = f2_pack(sl2, sl2), nmx2 = f2_pack(-m, -m);
+      // (MASKED) while every key seen so far was excluded, m is -inf: use 0 so p = 2^-inf = 0
+      const float nm = (MASKED && m == -INFINITY) ? 0.f : -m;
+      const uint64_t sl2x2 = f2_pack(sl2, sl2), nmx2 = f2_pack(nm, nm);
       uint64_t l4[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
@@ -481,14 +590,16 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       tc_fence_before();
       mbar_arrive(bar(C::kBarPFull + X));
     }
-    // epilogue
-    if (!__all_sync(0xffffffffu,
-                    mbar_wait(bar(C::kBarODone + X), o_cnt & 1, abort, kWaitLimitNs))) {
-      flag_error(p, 4);
-      return;
+    // epilogue (an empty unit has no accumulator to wait for: l == 0 writes zeros)
+    if (!empty_unit) {
+      if (!__all_sync(0xffffffffu,
+                      mbar_wait(bar(C::kBarODone + X), o_cnt & 1, abort, kWaitLimitNs))) {
+        flag_error(p, 4);
+        return;
+      }
+      ++o_cnt;
+      tc_fence_after();
     }
-    ++o_cnt;
-    tc_fence_after();
     const int r = t * BM + row;
     bool valid = r < sc.R;
     int64_t token = 0;
@@ -499,17 +610,25 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
     }
     uint16_t* orow = p.O + token * p.o_row_stride + static_cast<int64_t>(u.h) * D;
     if (u.part < 0) {
-      // whole item: O / l -> bf16
-      const float inv_l = 1.0f / l;
+      // whole item: O / l -> bf16.  A row that may attend to no key gets O = 0 and LSE = -inf;
+      // its accumulator may never have been written in this unit, so zeros are stored, not
+      // 0 * accumulator.
+      const bool none = MASKED && l == 0.f;
+      const float inv_l = none ? 0.f : 1.0f / l;
 #pragma unroll 1
       for (int c = 0; c < D / 32; ++c) {
         uint32_t o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_wait_ld();
+        if (none) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = 0u;
+        }
         if (valid) store_row_bf16<32>(orow + c * 32, reinterpret_cast<const float*>(o), inv_l);
       }
       if (valid && p.lse)
-        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] = (m + __log2f(l)) * 0.69314718055994531f;
+        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] =
+            (MASKED && l == 0.f) ? -INFINITY : (m + __log2f(l)) * 0.69314718055994531f;
       continue;
     }
     // split item: publish this KV range's partial row, then the last range to finish merges
@@ -520,10 +639,13 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       tmem_ld32(tO + c * 32, o);
       tmem_wait_ld();
       float4* dst = reinterpret_cast<float4*>(part + c * 32);
+      const bool none = MASKED && l == 0.f;  // no allowed key in this range: O is not written
 #pragma unroll
       for (int q = 0; q < 8; ++q)
-        __stcg(dst + q, make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
-                                    __uint_as_float(o[4 * q + 2]), __uint_as_float(o[4 * q + 3])));
+        __stcg(dst + q, none ? make_float4(0.f, 0.f, 0.f, 0.f)
+                             : make_float4(__uint_as_float(o[4 * q]), __uint_as_float(o[4 * q + 1]),
+                                           __uint_as_float(o[4 * q + 2]),
+                                           __uint_as_float(o[4 * q + 3])));
     }
     __stcg(reinterpret_cast<float4*>(part + D), make_float4(m, l, 0.f, 0.f));
     __threadfence();
@@ -554,9 +676,10 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       float L = 0.f;
       for (int c = 0; c < sc.C; ++c) {
         const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + c * stride + D));
-        L += ml.y * ex2_approx(ml.x - M);
+        if (!(MASKED && M == -INFINITY)) L += ml.y * ex2_approx(ml.x - M);
       }
-      const float inv_L = 1.0f / L;
+      const bool empty = MASKED && M == -INFINITY;  // no range saw an allowed key
+      const float inv_L = empty ? 0.f : 1.0f / L;
 #pragma unroll 1
       for (int cc = 0; cc < D / 32; ++cc) {
         float acc[32];
@@ -564,7 +687,7 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         for (int e = 0; e < 32; ++e) acc[e] = 0.f;
         for (int c = 0; c < sc.C; ++c) {
           const float* pc = base + c * stride;
-          const float wgt = ex2_approx(__ldcg(pc + D) - M);
+          const float wgt = empty ? 0.f : ex2_approx(__ldcg(pc + D) - M);
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             const float4 v = __ldcg(reinterpret_cast<const float4*>(pc + cc * 32) + q);
@@ -577,13 +700,14 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         store_row_bf16<32>(orow + cc * 32, acc, inv_L);
       }
       if (p.lse)
-        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] = (M + __log2f(L)) * 0.69314718055994531f;
+        p.lse[static_cast<int64_t>(u.h) * p.S_tok + token] =
+            empty ? -INFINITY : (M + __log2f(L)) * 0.69314718055994531f;
     }
     if (row == 0) p.ws_count[2 * u.item + X] = 0;  // ready for the next launch
   }
 }
 
-template <int D>
+template <int D, bool MASKED>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const AttnParams p) {
@@ -636,16 +760,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp < 4) {
     reg_dealloc<kRegsControl>();
     if (warp == 0) {
-      if (lane == 0) producer<D>(&tmQ, &tmK, &tmV, p, sc, sQ0, sKV0, bar0, abort);
+      if (lane == 0) producer<D, MASKED>(&tmQ, &tmK, &tmV, p, sc, sQ0, sKV0, bar0, abort);
       __syncwarp();
     } else if (warp == 1) {
-      if (lane == 0) mma_issuer<D>(p, sc, tmem, sQ0, sKV0, bar0, abort);
+      if (lane == 0) mma_issuer<D, MASKED>(p, sc, tmem, sQ0, sKV0, bar0, abort);
       __syncwarp();
     }
   } else {
     reg_alloc<kRegsSoftmax>();
     const int X = (warp - 4) >> 2;
-    softmax_group<D>(p, sc, X, tmem, bar0, abort, merge_flag + 2 * X);
+    softmax_group<D, MASKED>(p, sc, X, tmem, bar0, abort, merge_flag + 2 * X);
   }
 
   tc_fence_before();
@@ -701,7 +825,7 @@ int64_t workspace_bytes(int d, int grid) {
   return kCountBytes + static_cast<int64_t>(grid) * 2 * BM * (d + 4) * 4;
 }
 
-template <int D>
+template <int D, bool MASKED>
 rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
                  const AttnParams& p, int grid, const DeviceInfo& di, cudaStream_t stream) {
   using C = Cfg<D>;
@@ -709,11 +833,11 @@ rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& 
   if (C::kSmemBytes > di.max_smem_optin) return fail(RF_ERR_UNSUPPORTED, "shared memory");
   if (!attr_set[di.device]) {
     if (cudaError_t e = cudaFuncSetAttribute(
-            attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes))
+            attn_kernel<D, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes))
       return fail(RF_ERR_CUDA, "cudaFuncSetAttribute(attn_kernel)", e);
     attr_set[di.device] = true;
   }
-  attn_kernel<D><<<grid, kThreads, C::kSmemBytes, stream>>>(q, k, v, p);
+  attn_kernel<D, MASKED><<<grid, kThreads, C::kSmemBytes, stream>>>(q, k, v, p);
   return launch_status("attn_kernel launch");
 }
 
@@ -740,12 +864,12 @@ extern "C" int64_t rf_attn_workspace_bytes(int d) {
   return workspace_bytes(d, grid);
 }
 
-extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
-                             const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride, int F,
-                             int N, int H, int d, const int32_t* d_active,
-                             const int32_t* d_counts, float softmax_scale, void* d_workspace,
-                             int64_t workspace_bytes_given, int32_t* d_status,
-                             rf_stream_t stream) {
+namespace {
+rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, const void* d_V,
+                    int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H, int d,
+                    const int32_t* d_active, const int32_t* d_counts, float softmax_scale,
+                    const uint8_t* d_block_mask, void* d_workspace, int64_t workspace_bytes_given,
+                    int32_t* d_status, rf_stream_t stream) {
   if (!d_O || !d_Q || !d_K || !d_V || !d_active || !d_counts) return RF_ERR_INVALID_ARG;
   if (F < 1 || N < 1 || H < 1 || H > 65535) return RF_ERR_INVALID_ARG;
   if (d != 64 && d != 128) return RF_ERR_UNSUPPORTED;
@@ -791,6 +915,7 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   p.ws_count = split ? static_cast<int*>(d_workspace) : nullptr;
   p.ws_part = split ? reinterpret_cast<float*>(static_cast<char*>(d_workspace) + kCountBytes)
                     : nullptr;
+  p.block_mask = d_block_mask;
   p.o_row_stride = o_row_stride;
   p.F = F;
   p.N = N;
@@ -800,7 +925,37 @@ extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const voi
   p.nkv = static_cast<int>((S_tok + BN - 1) / BN);
   p.scale_log2 = static_cast<float>(static_cast<double>(softmax_scale) * 1.4426950408889634);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  return d == 128 ? launch<128>(mq, mk, mv, p, grid, di, s) : launch<64>(mq, mk, mv, p, grid, di, s);
+  if (d_block_mask)
+    return d == 128 ? launch<128, true>(mq, mk, mv, p, grid, di, s)
+                    : launch<64, true>(mq, mk, mv, p, grid, di, s);
+  return d == 128 ? launch<128, false>(mq, mk, mv, p, grid, di, s)
+                  : launch<64, false>(mq, mk, mv, p, grid, di, s);
+}
+}  // namespace
+
+extern "C" rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
+                             const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride, int F,
+                             int N, int H, int d, const int32_t* d_active,
+                             const int32_t* d_counts, float softmax_scale, void* d_workspace,
+                             int64_t workspace_bytes_given, int32_t* d_status,
+                             rf_stream_t stream) {
+  return attn_impl(d_O, d_lse, d_Q, d_K, d_V, qkv_row_stride, o_row_stride, F, N, H, d, d_active,
+                   d_counts, softmax_scale, nullptr, d_workspace, workspace_bytes_given, d_status,
+                   stream);
+}
+
+extern "C" rf_status rf_attn_block_masked(void* d_O, float* d_lse, const void* d_Q,
+                                          const void* d_K, const void* d_V,
+                                          int64_t qkv_row_stride, int64_t o_row_stride, int F,
+                                          int N, int H, int d, const int32_t* d_active,
+                                          const int32_t* d_counts, float softmax_scale,
+                                          const uint8_t* d_block_mask, void* d_workspace,
+                                          int64_t workspace_bytes_given, int32_t* d_status,
+                                          rf_stream_t stream) {
+  if (!d_block_mask) return RF_ERR_INVALID_ARG;
+  return attn_impl(d_O, d_lse, d_Q, d_K, d_V, qkv_row_stride, o_row_stride, F, N, H, d, d_active,
+                   d_counts, softmax_scale, d_block_mask, d_workspace, workspace_bytes_given,
+                   d_status, stream);
 }
 
 // rf_attn without any device allocation: the split-KV scratch is the library's own static

@@ -548,3 +548,93 @@ def test_graph_replay_matches_eager(cuda_lib, name):
     assert torch.equal(cg.z2, eager.z2)
     assert torch.equal(O1, O2)
     assert cg.status.item() == 0
+
+
+# ---------------------------------------------------------------------------
+# rf_attn_block_masked: frame mask x token block mask (Appendix D)
+# ---------------------------------------------------------------------------
+def _run_masked(rf, Q, K, V, F, N, mask, scale, bmask, split=True):
+    H, d = Q.shape[1], Q.shape[2]
+    S_tok = F * N
+    O = torch.full((S_tok, H, d), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    L = torch.full((H, S_tok), SENTINEL, dtype=torch.float32, device=DEV)
+    act = torch.zeros(F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(torch.as_tensor(np.asarray(mask, np.uint8)).to(DEV), F, N, act, skp,
+                           None, cnt)
+    ws = _workspace(rf, d) if split else None
+    rf.rf_attn_block_masked(O, L, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt, scale,
+                            torch.from_numpy(bmask).to(DEV), ws, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    if ws is not None:
+        assert int(ws[:1024].abs().sum()) == 0
+    return O, L
+
+
+def _check_masked(Q, K, V, O, L, mask, N, scale, bmask, label):
+    rows = _active_rows(mask, N)
+    Oref, Lref = oracle.attention_block_masked(Q.cpu(), K.cpu(), V.cpu(), rows, scale, bmask)
+    Og = O.cpu().float()[rows].numpy()
+    Lg = L.cpu()[:, rows].numpy()
+    empty = np.isneginf(Lref)                      # [H, rows]: no allowed key
+    assert (Og.transpose(1, 0, 2)[empty] == 0).all(), label
+    assert np.isneginf(Lg[empty]).all(), label
+    keep = ~empty.any(axis=0)
+    if keep.any():
+        compare(Og[keep], Oref[keep], Lg[:, keep], Lref[:, keep], label)
+    skipped = sorted(set(range(len(mask) * N)) - set(rows))
+    if skipped:
+        assert (O.cpu()[torch.tensor(skipped[:4096])].float() == SENTINEL).all()
+
+
+@pytest.mark.parametrize("F,N,H,d,mask,density,split", [
+    (4, 256, 2, 128, [1, 1, 1, 1], 0.5, True),
+    (4, 256, 2, 128, [1, 0, 0, 1], 0.3, False),
+    (5, 100, 2, 64, [1, 0, 1, 1, 0], 0.6, True),     # N % 8 != 0
+    (3, 1560, 2, 128, [1, 0, 1], 0.4, True),         # ragged KV tail, several tiles per frame
+    (3, 1560, 2, 128, [1, 1, 1], 0.15, False),
+])
+def test_attn_block_masked_parity(cuda_lib, F, N, H, d, mask, density, split):
+    rf = cuda_lib
+    Q, K, V = _qkv(F * N, H, d, seed=F * 31 + N + d)
+    nb = (F * N + 127) // 128
+    rng = np.random.default_rng(F + N + int(100 * density))
+    bm = (rng.random((H, nb, nb)) < density).astype(np.uint8)
+    bm[:, 0, :] = 0                                  # query block 0 may attend to nothing
+    scale = 1.0 / math.sqrt(d)
+    O, L = _run_masked(rf, Q, K, V, F, N, mask, scale, bm, split)
+    _check_masked(Q, K, V, O, L, mask, N, scale, bm, f"{F}x{N} d{d} {mask} p={density}")
+
+
+def test_attn_block_masked_all_allowed_equals_unmasked(cuda_lib):
+    rf = cuda_lib
+    F, N, H, d = 3, 1560, 2, 128
+    Q, K, V = _qkv(F * N, H, d, seed=77)
+    nb = (F * N + 127) // 128
+    ones = np.ones((H, nb, nb), np.uint8)
+    O1, L1 = _run_masked(rf, Q, K, V, F, N, [1, 0, 1], 0.088, ones)
+    O2, L2 = _run_attn(rf, Q, K, V, F, N, [1, 0, 1], 0.088)
+    assert (O1.float() - O2.float()).abs().max().item() < 1e-2
+    rows = _active_rows([1, 0, 1], N)
+    assert (L1[:, rows] - L2[:, rows]).abs().max().item() < 1e-3
+
+
+def test_attn_block_masked_local_window_and_empty_items(cuda_lib):
+    """A local-window mask (each query block sees key blocks within +-2) and a head whose
+    mask is empty everywhere (every work item of that head has no key tile at all)."""
+    rf = cuda_lib
+    F, N, H, d = 5, 512, 2, 128
+    Q, K, V = _qkv(F * N, H, d, seed=5)
+    nb = (F * N + 127) // 128
+    qb, kb = np.meshgrid(np.arange(nb), np.arange(nb), indexing="ij")
+    bm = np.zeros((H, nb, nb), np.uint8)
+    bm[0] = (np.abs(qb - kb) <= 2)
+    mask = [1, 0, 1, 0, 1]
+    for split in (True, False):
+        O, L = _run_masked(rf, Q, K, V, F, N, mask, 1 / math.sqrt(d), bm, split)
+        _check_masked(Q, K, V, O, L, mask, N, 1 / math.sqrt(d), bm, f"window split={split}")
+        rows = _active_rows(mask, N)
+        assert (O[rows, 1].float() == 0).all() and torch.isneginf(L[1, rows]).all()

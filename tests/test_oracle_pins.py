@@ -382,3 +382,44 @@ def test_kv_cache_commutes_with_affine_map():
     zp = oracle.project(z[1 - slot, idx].reshape(F, -1), z[slot, idx].reshape(F, -1), alpha)
     want = zp.reshape(F, N, C) @ W + b
     np.testing.assert_allclose(out[:3], want[:3], rtol=0, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Frame mask x token block mask (Appendix D, combined mask)
+# --------------------------------------------------------------------------
+def test_block_masked_attention_matches_sdpa_with_mask():
+    """The element-wise product of the frame mask (rows = active frames' tokens) and a token
+    block mask equals torch SDPA with the expanded boolean mask, row by row."""
+    g = torch.Generator().manual_seed(9)
+    F, N, H, d, blk = 4, 48, 2, 16, 32
+    S_tok = F * N
+    Q, K, V = (torch.randn(S_tok, H, d, generator=g).to(torch.bfloat16) for _ in range(3))
+    nb = (S_tok + blk - 1) // blk
+    rng = np.random.default_rng(9)
+    bm = (rng.random((H, nb, nb)) < 0.5).astype(np.uint8)
+    bm[:, np.arange(nb), np.arange(nb)] = 1           # every query block sees itself
+    frame_mask = [1, 0, 1, 1]
+    rows = [f * N + p for f in range(F) if frame_mask[f] for p in range(N)]
+    O, L = oracle.attention_block_masked(Q, K, V, rows, 0.3, bm, block=blk)
+    tok_blk = np.arange(S_tok) // blk
+    full = torch.from_numpy(bm[:, tok_blk][:, :, tok_blk] != 0)            # [H, S, S]
+    q, k, v = (x.double().permute(1, 0, 2) for x in (Q, K, V))
+    ref = torch.nn.functional.scaled_dot_product_attention(q, k, v, attn_mask=full, scale=0.3)
+    np.testing.assert_allclose(O, ref.permute(1, 0, 2).numpy()[rows], rtol=0, atol=1e-12)
+    s = 0.3 * q @ k.transpose(1, 2)
+    lse = torch.logsumexp(s.masked_fill(~full, -np.inf), dim=-1)
+    np.testing.assert_allclose(L, lse.numpy()[:, rows], rtol=0, atol=1e-12)
+
+
+def test_block_masked_attention_all_allowed_is_dense_and_empty_rows_zero():
+    g = torch.Generator().manual_seed(10)
+    Q, K, V = (torch.randn(100, 1, 8, generator=g) for _ in range(3))
+    ones = np.ones((1, 4, 4), np.uint8)
+    O1, L1 = oracle.attention_block_masked(Q, K, V, range(100), 0.5, ones, block=32)
+    O2, L2 = oracle.attention(Q, K, V, range(100), 0.5)
+    np.testing.assert_allclose(O1, O2, rtol=0, atol=1e-13)
+    none = np.zeros((1, 4, 4), np.uint8)
+    none[0, 1] = 1                                      # only query block 1 sees anything
+    O3, L3 = oracle.attention_block_masked(Q, K, V, [5, 40, 99], 0.5, none, block=32)
+    assert (O3[[0, 2]] == 0).all() and np.isneginf(L3[0, [0, 2]]).all()
+    np.testing.assert_allclose(O3[1], O2[40], rtol=0, atol=1e-13)
