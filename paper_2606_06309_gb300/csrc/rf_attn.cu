@@ -6,9 +6,11 @@
 //     O[f*N+p, h, :] = softmax_j(scale * q . k_j) V_j     over all F*N tokens j.
 //
 // Design (one persistent CTA per SM, 384 threads, warp-specialised):
-//   warp 0      TMA producer: gathers the two query tiles of a work item by frame index
-//               (8-row boxes, so a tile can span several active frames) and streams K/V
-//               tiles of 128 tokens through a ring of shared-memory slots.
+//   warp 0      TMA producer: loads the two query tiles of a work item (one 128-row box
+//               when the tile lies in one active frame, else gathered by frame index in
+//               8-row boxes) and streams K/V tiles of 128 tokens through a ring of
+//               shared-memory slots.
+//   warp 2      (block-masked launches) builds each work item's list of KV tiles.
 //   warp 1      owns TMEM (512 columns) and one lane issues every tcgen05.mma:
 //               S = Q K^T (both operands in shared memory) and O += P V (P in TMEM).
 //   warps 4-7   softmax for query tile A, warps 8-11 for query tile B: thread = query row;
@@ -38,6 +40,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -62,6 +65,12 @@ constexpr uint64_t kDrainLimitNs = 200000000ull;  // 0.2 s for in-flight copies 
 constexpr float kRescaleLog2 = 8.0f;
 constexpr int kMaxSplit = 16;          // KV ranges per split item
 constexpr int kMaxGrid = 1024;         // workspace is sized for at most this many CTAs
+// Block-masked launches: a ring of per-unit KV-tile bitmaps in shared memory, one bit per KV
+// tile (so at most kTLWords * 32 tiles of 128 keys), followed by the number of set bits.
+constexpr int kTLSlots = 4;
+constexpr int kTLWords = 128;
+constexpr int kTLSlotBytes = kTLWords * 4 + 16;
+constexpr int kTLMaxTiles = kTLWords * 32;
 
 template <int D>
 struct Cfg {
@@ -81,6 +90,10 @@ struct Cfg {
   // misc: tmem address, abort flag, merge flags [2 groups][2 alternating slots]
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 32 + 1024;  // + slack to align the base
+  // (MASKED) tile-list ring: barriers tl_full[kTLSlots] tl_empty[kTLSlots], then the slots
+  static constexpr int kOffTL = (kOffMisc + 32 + 15) / 16 * 16;
+  static constexpr int kOffTLSlot = kOffTL + 2 * kTLSlots * 8;
+  static constexpr int kSmemBytesMasked = kOffTLSlot + kTLSlots * kTLSlotBytes + 1024;
   // split-KV partial row: D unnormalised outputs, running max (log2 units), running sum
   static constexpr int kPartFloats = D + 4;
 };
@@ -94,6 +107,8 @@ struct AttnParams {
   int* ws_count;   // [kMaxGrid] merge counters (zero between launches), or null: no split
   float* ws_part;  // [kMaxGrid][2][BM][D+4] partial rows
   const uint8_t* block_mask;  // [H][nkv][nkv] token block mask (128-token blocks), or null
+  const int* lpt_order;       // (block mask, with a workspace) unit order for the queue, or null
+  int lpt_group;              // heads per group of that order
   int64_t o_row_stride;
   int F, N, Np, H, S_tok, nkv;
   float scale_log2;
@@ -125,7 +140,10 @@ __device__ __forceinline__ Sched make_sched(const AttnParams& p) {
   const int G = gridDim.x;
   s.T_full = T;
   s.C = 1;
-  if (T > 0 && p.ws_count != nullptr) {
+  // Block-masked launches never split: their items differ in cost, so the makespan of the
+  // static assignment is set by the costliest CTA rather than by the last round's tail, and a
+  // split only adds the merge (measured slower on the 13 x 1560-token workload).
+  if (T > 0 && p.ws_count != nullptr && p.block_mask == nullptr) {
     const int rounds = (T + G - 1) / G;
     const int tail = T - (rounds - 1) * G;
     int c = G / tail;
@@ -206,22 +224,33 @@ __device__ __forceinline__ QRanges unit_qranges(const AttnParams& p, const Sched
   return q;
 }
 
-// May any query block of the unit attend to key block j?
-__device__ __forceinline__ bool unit_allows(const AttnParams& p, const QRanges& q, int j) {
-  for (int i = 0; i < q.n; ++i)
-    for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb)
-      if (q.mh[static_cast<int64_t>(qb) * p.nkv + j]) return true;
-  return false;
+// First set bit at or after j in a unit's tile bitmap of nw words; nw * 32 (>= nkv) if none.
+__device__ __forceinline__ int next_kept(const uint32_t* words, int j, int nw) {
+  int wi = j >> 5;
+  if (wi >= nw) return nw << 5;
+  uint32_t x = words[wi] & (0xFFFFFFFFu << (j & 31));
+  while (x == 0) {
+    if (++wi >= nw) return nw << 5;
+    x = words[wi];
+  }
+  return (wi << 5) + __ffs(x) - 1;
 }
 
-// First allowed KV tile at or after j (u.j1 if none).
+// The KV tiles a role visits for a unit: [j0, j1) unmasked, the builder's bitmap when MASKED.
 template <bool MASKED>
-__device__ __forceinline__ int next_tile(const AttnParams& p, const QRanges& q, const Unit& u,
-                                         int j) {
-  if constexpr (MASKED) {
-    while (j < u.j1 && !unit_allows(p, q, j)) ++j;
-  }
-  return j;
+__device__ __forceinline__ int tile_first(const Unit& u, const uint32_t* tw, int nw) {
+  if constexpr (MASKED) return next_kept(tw, 0, nw);
+  else return u.j0;
+}
+template <bool MASKED>
+__device__ __forceinline__ int tile_next(const uint32_t* tw, int nw, int j) {
+  if constexpr (MASKED) return next_kept(tw, j + 1, nw);
+  else return j + 1;
+}
+template <bool MASKED>
+__device__ __forceinline__ int tile_end(const Unit& u, const AttnParams& p) {
+  if constexpr (MASKED) return p.nkv;
+  else return u.j1;
 }
 
 __device__ __forceinline__ void flag_error(const AttnParams& p, int where) {
@@ -245,22 +274,139 @@ __device__ __forceinline__ bool group_sync(uint32_t bar, int& cnt, volatile int*
   return ok;
 }
 
+// (MASKED) The tile-list ring in shared memory: slot k % kTLSlots holds the KV-tile bitmap of
+// the CTA's k-th unit and, after kTLWords words, its number of set bits.
+struct TLRing {
+  uint32_t bar;     // shared address of tl_full[0]; tl_empty[s] follows the kTLSlots full barriers
+  uint32_t* slots;  // slot 0
+  __device__ __forceinline__ uint32_t full(int k) const { return bar + 8u * (k % kTLSlots); }
+  __device__ __forceinline__ uint32_t empty(int k) const {
+    return bar + 8u * (kTLSlots + k % kTLSlots);
+  }
+  __device__ __forceinline__ uint32_t* words(int k) const {
+    return slots + (k % kTLSlots) * (kTLSlotBytes / 4);
+  }
+  __device__ __forceinline__ int parity(int k) const { return (k / kTLSlots) & 1; }
+  // the unit the slot describes, or -1: the CTA has no more units
+  __device__ __forceinline__ int unit(int k) const {
+    return static_cast<int>(words(k)[kTLWords + 1]);
+  }
+};
+// Arrivals that release a slot: the producer, the MMA issuer and the 256 softmax threads.
+constexpr int kTLConsumers = 2 + 256;
+// (MASKED, with a workspace) work-queue words in the workspace's counter area, which split-KV
+// would use but block-masked launches never split: the next unit to hand out, and the number
+// of CTAs done.  The last CTA to finish sets both back to zero.
+constexpr int kQueueNext = 0, kQueueDone = 1;
+
+// ---------------------------------------------------------------------------------------
+// Tile-list builder (MASKED only; warp 2, all 32 lanes).
+// ---------------------------------------------------------------------------------------
+// For every unit of this CTA, in order, one ring slot receives the bitmap of the KV tiles the
+// unit visits: the tiles some query block of its rows may attend to (block-masked launches
+// never split, so a unit is a whole item).  The other roles walk this bitmap, so the block
+// mask in global memory is scanned once per unit, with 32 lanes loading independent bytes,
+// instead of tile by tile on the critical paths of the producer and the MMA issuer.
+__device__ __forceinline__ void tile_list_builder(const AttnParams& p, const Sched& sc,
+                                                  const TLRing& tl, volatile int* abort) {
+  const int lane = threadIdx.x & 31;
+  const int nw = (p.nkv + 31) >> 5;
+  for (int k = 0;; ++k) {
+    // At most two units in flight per CTA: the one being processed and the next.  A unit
+    // taken from the queue long before it is processed would unbalance the end of the launch.
+    // Unit k - 2 released also means slot k's previous unit, k - 4, was released.
+    if (k >= 2 && !__all_sync(0xffffffffu, mbar_wait(tl.empty(k - 2), tl.parity(k - 2), abort,
+                                                     kWaitLimitNs))) {
+      if (lane == 0) flag_error(p, 7);
+      return;
+    }
+    // with a workspace: the next unit of the queue shared by all CTAs (greedy list
+    // scheduling: items differ in cost under a mask); without: the static round-robin deal
+    int w;
+    if (p.ws_count != nullptr) {
+      int t = 0;
+      if (lane == 0) {
+        t = atomicAdd(p.ws_count + kQueueNext, 1);
+        if (p.lpt_order != nullptr && t < sc.units) t = p.lpt_order[t];
+      }
+      w = __shfl_sync(0xffffffffu, t, 0);
+    } else {
+      w = blockIdx.x + k * static_cast<int>(gridDim.x);
+    }
+    uint32_t* words = tl.words(k);
+    if (w >= sc.units) {
+      if (lane == 0) {
+        words[kTLWords] = 0u;
+        words[kTLWords + 1] = 0xFFFFFFFFu;
+      }
+      mbar_arrive(tl.full(k));
+      return;
+    }
+    const Unit u = get_unit(sc, p, w);
+    const QRanges q = unit_qranges(p, sc, u);
+    int total = 0;
+    for (int k0 = 0; k0 < nw; k0 += 32) {
+      // bit l of acc: may some query block of the unit attend to tile (k0 + l) * 32 + lane?
+      uint32_t acc = 0;
+      for (int i = 0; i < q.n; ++i)
+        for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb) {
+          const uint8_t* mrow = q.mh + static_cast<int64_t>(qb) * p.nkv;
+#pragma unroll
+          for (int l = 0; l < 32; ++l) {
+            const int j = (k0 + l) * 32 + lane;
+            if (j < p.nkv && mrow[j] != 0) acc |= 1u << l;
+          }
+        }
+      // transpose: lane l collects word k0 + l (tiles (k0 + l) * 32 .. + 31)
+      uint32_t mine = 0;
+#pragma unroll
+      for (int l = 0; l < 32; ++l) {
+        const uint32_t bits = __ballot_sync(0xffffffffu, (acc >> l) & 1u);
+        if (lane == l) mine = bits;
+      }
+      if (k0 + lane < nw) words[k0 + lane] = mine;
+      total += __popc(mine);  // zero for words past nw: their tiles are >= nkv
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) total += __shfl_xor_sync(0xffffffffu, total, off);
+    if (lane == 0) {
+      words[kTLWords] = static_cast<uint32_t>(total);
+      words[kTLWords + 1] = static_cast<uint32_t>(w);
+    }
+    mbar_arrive(tl.full(k));  // every lane (count 32) releases its own stores
+  }
+}
+
 // ---------------------------------------------------------------------------------------
 // TMA producer (one thread).
 // ---------------------------------------------------------------------------------------
 template <int D, bool MASKED>
-__device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorMap* tmK,
+__device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorMap* tmQ128,
+                                         const CUtensorMap* tmK,
                                          const CUtensorMap* tmV, const AttnParams& p,
                                          const Sched& sc, uint32_t sQ0, uint32_t sKV0,
-                                         uint32_t bar0, volatile int* abort) {
+                                         uint32_t bar0, const TLRing& tl, volatile int* abort) {
   using C = Cfg<D>;
   auto bar = [&](int i) { return bar0 + 8u * i; };
+  const int nw = (p.nkv + 31) >> 5;
   int q_cnt[2] = {0, 0};
   int it = 0;
-  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+  for (int k = 0;; ++k) {  // k: units so far (MASKED: tile-list ring position)
+    int w;
+    const uint32_t* tw = nullptr;
+    if constexpr (MASKED) {
+      if (!mbar_wait(tl.full(k), tl.parity(k), abort, kWaitLimitNs)) {
+        flag_error(p, 0);
+        goto drain;
+      }
+      w = tl.unit(k);
+      if (w < 0) break;
+      tw = tl.words(k);
+    } else {
+      w = blockIdx.x + k * static_cast<int>(gridDim.x);
+      if (w >= sc.units) break;
+    }
     const Unit u = get_unit(sc, p, w);
-    QRanges qr{};
-    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
     for (int X = 0; X < 2; ++X) {
       const int t = 2 * u.pr + X;
       if (t >= sc.tiles) break;
@@ -270,24 +416,39 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
       }
       mbar_arrive_expect_tx(bar(C::kBarQFull + X), C::kTileBytes);
       const uint32_t dst = sQ0 + X * C::kTileBytes;
-#pragma unroll 1
-      for (int b = 0; b < BM / 8; ++b) {
-        const int r = t * BM + b * 8;
-        int tok = p.S_tok;  // rows past the active list: out of bounds, zero filled
-        if (r < sc.R) {
-          const int a = r / p.Np;
-          tok = p.active[a] * p.N + (r - a * p.Np);
-        }
+      const int r0 = t * BM;
+      const int a0 = r0 / p.Np;
+      if (a0 == (min(r0 + BM, sc.R) - 1) / p.Np) {
+        // every row of the tile in one frame: one 128-row box per half (rows past the frame or
+        // the active list read the following tokens, or zeros past the sequence; they are
+        // never stored)
+        const int tok = p.active[a0] * p.N + (r0 - a0 * p.Np);
 #pragma unroll
         for (int hb = 0; hb < C::kHalves; ++hb)
-          tma_load_3d(dst + hb * C::kHalfBytes + b * 1024, tmQ, bar(C::kBarQFull + X), hb * 64,
-                      u.h, tok);
+          tma_load_3d(dst + hb * C::kHalfBytes, tmQ128, bar(C::kBarQFull + X), hb * 64, u.h,
+                      tok);
+      } else {
+        // a tile across frames: gathered in boxes of 8 rows (frames are padded to 8 rows)
+        int tok[BM / 8];
+#pragma unroll
+        for (int b = 0; b < BM / 8; ++b) {
+          const int r = r0 + b * 8;
+          const int a = r / p.Np;
+          tok[b] = r < sc.R ? p.active[a] * p.N + (r - a * p.Np)
+                            : p.S_tok;  // past the active list: out of bounds, zero filled
+        }
+#pragma unroll
+        for (int b = 0; b < BM / 8; ++b)
+#pragma unroll
+          for (int hb = 0; hb < C::kHalves; ++hb)
+            tma_load_3d(dst + hb * C::kHalfBytes + b * 1024, tmQ, bar(C::kBarQFull + X),
+                        hb * 64, u.h, tok[b]);
       }
       ++q_cnt[X];
     }
 #pragma unroll 1
-    for (int j = next_tile<MASKED>(p, qr, u, u.j0); j < u.j1;
-         j = next_tile<MASKED>(p, qr, u, j + 1)) {
+    for (int j = tile_first<MASKED>(u, tw, nw); j < tile_end<MASKED>(u, p);
+         j = tile_next<MASKED>(tw, nw, j)) {
 #pragma unroll
       for (int kv = 0; kv < 2; ++kv) {
         const int s = it % C::kSlots, n = it / C::kSlots;
@@ -304,6 +465,7 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
         ++it;
       }
     }
+    if constexpr (MASKED) mbar_arrive(tl.empty(k));
   }
 drain:
   // every armed fill has all its copies issued; wait for the last fill of each buffer
@@ -340,7 +502,7 @@ __device__ __forceinline__ void mma_pv(uint32_t tO, uint32_t tP, uint64_t dV, ui
 template <int D, bool MASKED>
 __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc, uint32_t tmem,
                                            uint32_t sQ0, uint32_t sKV0, uint32_t bar0,
-                                           volatile int* abort) {
+                                           const TLRing& tl, volatile int* abort) {
   using C = Cfg<D>;
   auto bar = [&](int i) { return bar0 + 8u * i; };
   const uint32_t tS[2] = {tmem, tmem + 128};
@@ -366,13 +528,24 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     tc_fence_after();
     return ok;
   };
-  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+  const int nw = (p.nkv + 31) >> 5;
+  for (int k = 0;; ++k) {  // k: units so far (MASKED: tile-list ring position)
+    int w;
+    const uint32_t* tw = nullptr;
+    if constexpr (MASKED) {
+      if (!mbar_wait(tl.full(k), tl.parity(k), abort, kWaitLimitNs)) goto fail;
+      w = tl.unit(k);
+      if (w < 0) break;
+      tw = tl.words(k);
+    } else {
+      w = blockIdx.x + k * static_cast<int>(gridDim.x);
+      if (w >= sc.units) break;
+    }
     const Unit u = get_unit(sc, p, w);
     const bool hasB = 2 * u.pr + 1 < sc.tiles;
-    // KV tiles of the unit: all of [j0, j1), or (MASKED) the allowed ones, walked in order
-    QRanges qr{};
-    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
-    int jc = next_tile<MASKED>(p, qr, u, u.j0);
+    // KV tiles of the unit: all of [j0, j1), or (MASKED) the bits of the builder's bitmap
+    int jc = u.j0;
+    if constexpr (MASKED) jc = next_kept(tw, 0, nw);
     if (!mbar_wait(bar(C::kBarQFull + 0), q_cnt[0] & 1, abort, kWaitLimitNs)) goto fail;
     ++q_cnt[0];
     if (hasB) {
@@ -380,10 +553,11 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       ++q_cnt[1];
     }
     tc_fence_after();
-    if (MASKED && jc >= u.j1) {
+    if (MASKED && jc >= p.nkv) {
       // no allowed key block: release the queries.  No output barrier is committed: the
       // softmax warps see the same empty tile list and write their result without waiting
       // (a commit here could run two phases ahead of them).
+      mbar_arrive(tl.empty(k));
       tc_commit(bar(C::kBarQEmpty + 0));
       if (hasB) tc_commit(bar(C::kBarQEmpty + 1));
       continue;
@@ -404,8 +578,8 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
 #pragma unroll 1
     for (int j = 0;; ++j) {
       if constexpr (MASKED) {
-        jc = next_tile<MASKED>(p, qr, u, jc + 1);
-        if (jc >= u.j1) break;
+        jc = next_kept(tw, jc + 1, nw);
+        if (jc >= p.nkv) break;
       } else {
         if (j + 1 >= u.j1 - u.j0) break;
       }
@@ -427,6 +601,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       if (!wait_p(0)) goto fail;
       mma_pv<D>(tO[0], tS[0], dV(sV), 1);
     }
+    if constexpr (MASKED) mbar_arrive(tl.empty(k));
     tc_commit(bar(C::kBarODone + 0));
     tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
@@ -465,8 +640,8 @@ __device__ __forceinline__ void store_row_bf16(uint16_t* orow, const float* o, f
 
 template <int D, bool MASKED>
 __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& sc, int X,
-                                              uint32_t tmem, uint32_t bar0, volatile int* abort,
-                                              volatile int* merge_flag) {
+                                              uint32_t tmem, uint32_t bar0, const TLRing& tl,
+                                              volatile int* abort, volatile int* merge_flag) {
   using C = Cfg<D>;
   auto bar = [&](int i) { return bar0 + 8u * i; };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -476,14 +651,32 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
   const uint32_t tS = tmem + lane_base + X * 128;
   const uint32_t tO = tmem + lane_base + 256 + X * 128;
   const float sl2 = p.scale_log2;
+  const int nw = (p.nkv + 31) >> 5;
   int s_cnt = 0, o_cnt = 0, g_cnt = 0, split_cnt = 0;
-  for (int w = blockIdx.x; w < sc.units; w += gridDim.x) {
+  for (int k = 0;; ++k) {  // k: units so far (MASKED: tile-list ring position)
+    int w;
+    const uint32_t* tw = nullptr;
+    if constexpr (MASKED) {
+      // every softmax thread takes every unit's slot, also when its tile is absent, so the
+      // slot's release count is the same for all units
+      if (!__all_sync(0xffffffffu, mbar_wait(tl.full(k), tl.parity(k), abort, kWaitLimitNs))) {
+        flag_error(p, 8);
+        return;
+      }
+      w = tl.unit(k);
+      if (w < 0) break;
+      tw = tl.words(k);
+    } else {
+      w = blockIdx.x + k * static_cast<int>(gridDim.x);
+      if (w >= sc.units) break;
+    }
     const Unit u = get_unit(sc, p, w);
     const int t = 2 * u.pr + X;
-    if (t >= sc.tiles) continue;
-    QRanges qr{};
-    if constexpr (MASKED) qr = unit_qranges(p, sc, u);
-    const bool empty_unit = MASKED && next_tile<MASKED>(p, qr, u, u.j0) >= u.j1;
+    if (t >= sc.tiles) {
+      if constexpr (MASKED) mbar_arrive(tl.empty(k));
+      continue;
+    }
+    const bool empty_unit = MASKED && tw[kTLWords] == 0u;
     float m = -INFINITY, l = 0.f;
     // this row's query block (MASKED): rows past the active list or in frame padding are
     // never stored and need no mask
@@ -498,9 +691,17 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         }
       }
     }
+    // (MASKED) this row's mask entry for the tile, loaded one tile ahead of its use
+    int j = tile_first<MASKED>(u, tw, nw);
+    const int j_end = tile_end<MASKED>(u, p);
+    uint32_t mk = 1u;
+    if constexpr (MASKED) mk = (mrow != nullptr && j < j_end) ? mrow[j] : 1u;
+    bool first = true;
 #pragma unroll 1
-    for (int j = next_tile<MASKED>(p, qr, u, u.j0); j < u.j1;
-         j = next_tile<MASKED>(p, qr, u, j + 1)) {
+    while (j < j_end) {
+      const int jn = tile_next<MASKED>(tw, nw, j);
+      uint32_t mk_next = 1u;
+      if constexpr (MASKED) mk_next = (mrow != nullptr && jn < j_end) ? mrow[jn] : 1u;
       // the result is made warp-uniform: tcgen05.ld/st below are warp-collective
       if (!__all_sync(0xffffffffu, mbar_wait(bar(C::kBarSFull + X), s_cnt & 1, abort,
                                             kWaitLimitNs))) {
@@ -520,12 +721,6 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         for (int c = 0; c < BN; ++c)
           if (c >= valid) sf[c] = -INFINITY;
       }
-      if constexpr (MASKED) {
-        if (mrow != nullptr && mrow[j] == 0) {
-#pragma unroll
-          for (int c = 0; c < BN; ++c) sf[c] = -INFINITY;
-        }
-      }
       // row max: 8 independent chains of three-input maxima (a single 128-long chain of
       // two-input maxima is pure latency on the path from QK^T to PV)
       float mx8[8];
@@ -537,7 +732,8 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], sf[c + i], sf[c + 8 + i]);
       const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                              fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      const float m_new = fmaxf(m, mx * sl2);
+      // (MASKED) a tile this row may not see leaves its max alone (and gets p = 0 below)
+      const float m_new = fmaxf(m, (MASKED && mk == 0u) ? -INFINITY : mx * sl2);
       const bool need = m_new > m + kRescaleLog2;
       const bool rescale = __any_sync(0xffffffffu, need);
       float fac = 1.f;
@@ -550,8 +746,10 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       }
       // p = 2^(s*scale*log2(e) - m) with packed fp32 pairs for the scale/subtract and the
       // row sum (8 independent sum chains in 4 packed accumulators)
-      // (MASKED) while every key seen so far was excluded, m is -inf: use 0 so p = 2^-inf = 0
-      const float nm = (MASKED && m == -INFINITY) ? 0.f : -m;
+      // (MASKED) while every key seen so far was excluded, m is -inf: use 0 so p = 2^-inf = 0;
+      // for a tile the row may not see, an offset of -inf gives p = 0 for every key (s is
+      // finite or -inf, so s * scale - inf is -inf, never NaN)
+      const float nm = (MASKED && mk == 0u) ? -INFINITY : (MASKED && m == -INFINITY) ? 0.f : -m;
       const uint64_t sl2x2 = f2_pack(sl2, sl2), nmx2 = f2_pack(nm, nm);
       uint64_t l4[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
@@ -574,8 +772,9 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
         f2_unpack(t2, a, b);
         l += a + b;
       }
-      // O was last written by PV(j-1), which completed before S(j) was signalled
-      if (rescale && j > u.j0) {
+      // O was last written by the previous tile's PV, which completed before S(j) was
+      // signalled; at the unit's first tile it holds nothing yet
+      if (rescale && (MASKED ? !first : j > u.j0)) {
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           uint32_t o[32];
@@ -589,7 +788,11 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(bar(C::kBarPFull + X));
+      first = false;
+      j = jn;
+      mk = mk_next;
     }
+    if constexpr (MASKED) mbar_arrive(tl.empty(k));
     // epilogue (an empty unit has no accumulator to wait for: l == 0 writes zeros)
     if (!empty_unit) {
       if (!__all_sync(0xffffffffu,
@@ -709,7 +912,8 @@ __device__ __forceinline__ void softmax_group(const AttnParams& p, const Sched& 
 
 template <int D, bool MASKED>
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmQ128,
+                const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const AttnParams p) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -739,9 +943,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar0 + 8 * (C::kBarKVEmpty + s), 1);
     }
     mbar_init(bar0 + 8 * C::kBarDrain, 1);
+    if constexpr (MASKED) {
+      for (int s = 0; s < kTLSlots; ++s) {
+        mbar_init(sbase + C::kOffTL + 8 * s, 32);
+        mbar_init(sbase + C::kOffTL + 8 * (kTLSlots + s), kTLConsumers);
+      }
+    }
     *abort = 0;
     fence_mbar_init();
     tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmQ128);
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmV);
   }
@@ -754,22 +965,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const Sched sc = make_sched(p);
+  TLRing tl{};
+  if constexpr (MASKED)
+    tl = TLRing{sbase + C::kOffTL, reinterpret_cast<uint32_t*>(smem + C::kOffTLSlot)};
 
   // Every warp of warpgroup 0 gives registers back before any softmax warp asks for more,
   // so the increase below always finds them.
   if (warp < 4) {
     reg_dealloc<kRegsControl>();
     if (warp == 0) {
-      if (lane == 0) producer<D, MASKED>(&tmQ, &tmK, &tmV, p, sc, sQ0, sKV0, bar0, abort);
+      if (lane == 0) producer<D, MASKED>(&tmQ, &tmQ128, &tmK, &tmV, p, sc, sQ0, sKV0, bar0, tl, abort);
       __syncwarp();
     } else if (warp == 1) {
-      if (lane == 0) mma_issuer<D, MASKED>(p, sc, tmem, sQ0, sKV0, bar0, abort);
+      if (lane == 0) mma_issuer<D, MASKED>(p, sc, tmem, sQ0, sKV0, bar0, tl, abort);
       __syncwarp();
+    } else if (MASKED && warp == 2) {
+      tile_list_builder(p, sc, tl, abort);
     }
   } else {
     reg_alloc<kRegsSoftmax>();
     const int X = (warp - 4) >> 2;
-    softmax_group<D, MASKED>(p, sc, X, tmem, bar0, abort, merge_flag + 2 * X);
+    softmax_group<D, MASKED>(p, sc, X, tmem, bar0, tl, abort, merge_flag + 2 * X);
   }
 
   tc_fence_before();
@@ -778,6 +994,110 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  if constexpr (MASKED) {
+    // every CTA that reaches this point has taken its last unit from the queue; the last one
+    // to arrive leaves the queue words at zero for the next launch
+    if (threadIdx.x == 0 && p.ws_count != nullptr) {
+      __threadfence();
+      if (atomicAdd(p.ws_count + kQueueDone, 1) == static_cast<int>(gridDim.x) - 1) {
+        p.ws_count[kQueueNext] = 0;
+        p.ws_count[kQueueDone] = 0;
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// Longest-first order of block-masked work items (two small launches before the attention
+// kernel).  Under a mask, items differ in cost (the number of KV tiles their tile pair may
+// see); handing them out from the work queue longest first within each head (LPT list
+// scheduling) keeps the CTAs' finishing times close where a round-robin deal or the natural
+// order can leave costly items for the end (a causal block mask on 13 x 1560 tokens: 1.205 ms
+// dealt round-robin, 0.918 ms longest first).
+// ---------------------------------------------------------------------------------------
+// One warp per item: its cost is the number of set bits of the bitmap the builder will write.
+__global__ void __launch_bounds__(256) item_cost_kernel(const AttnParams p, int* cost) {
+  const Sched sc = make_sched(p);  // a block-masked launch: no split, so units are items
+  const int lane = threadIdx.x & 31;
+  const int item = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (item >= sc.units) return;
+  const Unit u = get_unit(sc, p, item);
+  const QRanges q = unit_qranges(p, sc, u);
+  int total = 0;
+  for (int j0 = 0; j0 < p.nkv; j0 += 32) {
+    const int j = j0 + lane;
+    bool ok = false;
+    if (j < p.nkv)
+      for (int i = 0; i < q.n; ++i)
+        for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb)
+          ok = ok || q.mh[static_cast<int64_t>(qb) * p.nkv + j] != 0;
+    total += __popc(__ballot_sync(0xffffffffu, ok));
+  }
+  if (lane == 0) cost[item] = total;
+}
+
+// One CTA per group of lpt_group consecutive heads: the group's items (item = head * pairs +
+// pair) by decreasing cost.  The queue hands out the groups one after the
+// other, so the CTAs that run together work on the heads of one group, whose K/V the host sized
+// to fit in L2: one global order by cost spread them over all 40 heads of a 21 x 3600-token
+// workload (39 MB of K/V per head, 129 MB of L2) and was 5% slower than no order at all.  The
+// host also makes a group hold several items per CTA, so that its costly items do not start
+// late: one head per group left 13 x 1560 tokens (80 items per head, 152 CTAs) 19% slower
+// than the global order.
+// A counting sort over the costs (at most kTLMaxTiles): the order among equal costs is
+// arbitrary, which changes no result (every item is computed the same way by whichever CTA
+// takes it).
+constexpr int kOrderThreads = 1024;
+constexpr int kBinsPerThread = (kTLMaxTiles + 1 + kOrderThreads - 1) / kOrderThreads;
+__global__ void __launch_bounds__(kOrderThreads) lpt_order_kernel(const AttnParams p,
+                                                                  const int* cost, int* order) {
+  __shared__ int start[kBinsPerThread * kOrderThreads];  // bin b holds cost kTLMaxTiles - b
+  __shared__ int warp_sum[kOrderThreads / 32];
+  const Sched sc = make_sched(p);
+  const int base = blockIdx.x * p.lpt_group * sc.pairs;
+  const int n = min(p.lpt_group * sc.pairs, sc.units - base);
+  if (n <= 0) return;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  for (int i = tid; i < kBinsPerThread * kOrderThreads; i += kOrderThreads) start[i] = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += kOrderThreads) atomicAdd(&start[kTLMaxTiles - cost[base + i]], 1);
+  __syncthreads();
+  // exclusive prefix sum over the bins: kBinsPerThread consecutive bins per thread, then a
+  // block-wide scan of the per-thread sums
+  int own[kBinsPerThread];
+  int sum = 0;
+#pragma unroll
+  for (int b = 0; b < kBinsPerThread; ++b) {
+    own[b] = start[tid * kBinsPerThread + b];
+    sum += own[b];
+  }
+  int incl = sum;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += t;
+  }
+  if (lane == 31) warp_sum[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    int v = warp_sum[lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, v, off);
+      if (lane >= off) v += t;
+    }
+    warp_sum[lane] = v;  // inclusive, over warps
+  }
+  __syncthreads();
+  int run = incl - sum + (wid > 0 ? warp_sum[wid - 1] : 0);
+#pragma unroll
+  for (int b = 0; b < kBinsPerThread; ++b) {
+    start[tid * kBinsPerThread + b] = run;
+    run += own[b];
+  }
+  __syncthreads();
+  for (int i = tid; i < n; i += kOrderThreads)
+    order[base + atomicAdd(&start[kTLMaxTiles - cost[base + i]], 1)] = base + i;
 }
 
 // ---------------------------------------------------------------------------------------
@@ -826,18 +1146,20 @@ int64_t workspace_bytes(int d, int grid) {
 }
 
 template <int D, bool MASKED>
-rf_status launch(const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v,
+rf_status launch(const CUtensorMap& q, const CUtensorMap& q128, const CUtensorMap& k,
+                 const CUtensorMap& v,
                  const AttnParams& p, int grid, const DeviceInfo& di, cudaStream_t stream) {
   using C = Cfg<D>;
+  constexpr int smem = MASKED ? C::kSmemBytesMasked : C::kSmemBytes;
   static bool attr_set[64] = {};
-  if (C::kSmemBytes > di.max_smem_optin) return fail(RF_ERR_UNSUPPORTED, "shared memory");
+  if (smem > di.max_smem_optin) return fail(RF_ERR_UNSUPPORTED, "shared memory");
   if (!attr_set[di.device]) {
     if (cudaError_t e = cudaFuncSetAttribute(
-            attn_kernel<D, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes))
+            attn_kernel<D, MASKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem))
       return fail(RF_ERR_CUDA, "cudaFuncSetAttribute(attn_kernel)", e);
     attr_set[di.device] = true;
   }
-  attn_kernel<D, MASKED><<<grid, kThreads, C::kSmemBytes, stream>>>(q, k, v, p);
+  attn_kernel<D, MASKED><<<grid, kThreads, smem, stream>>>(q, q128, k, v, p);
   return launch_status("attn_kernel launch");
 }
 
@@ -883,6 +1205,8 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
   if (qkv_row_stride % 8 != 0 || o_row_stride % 8 != 0) return RF_ERR_MISALIGNED;
   if (!aligned16(d_Q) || !aligned16(d_K) || !aligned16(d_V) || !aligned16(d_O))
     return RF_ERR_MISALIGNED;
+  if (d_block_mask && (S_tok + BN - 1) / BN > kTLMaxTiles)
+    return fail(RF_ERR_UNSUPPORTED, "block mask: more than 4096 key blocks of 128 tokens");
   if (d_workspace) {
     if (workspace_bytes_given < 0) return RF_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return RF_ERR_MISALIGNED;
@@ -891,8 +1215,10 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
   if (rf_status st = current_device_info(&di)) return st;
   if (di.cc_major != 10 || di.cc_minor != 3) return fail(RF_ERR_UNSUPPORTED, "needs sm_103");
 
-  CUtensorMap mq, mk, mv;
+  CUtensorMap mq, mq128, mk, mv;
   if (rf_status st = make_map(&mq, d_Q, d, H, static_cast<int>(S_tok), qkv_row_stride, 8)) return st;
+  if (rf_status st = make_map(&mq128, d_Q, d, H, static_cast<int>(S_tok), qkv_row_stride, BM))
+    return st;
   if (rf_status st = make_map(&mk, d_K, d, H, static_cast<int>(S_tok), qkv_row_stride, BN)) return st;
   if (rf_status st = make_map(&mv, d_V, d, H, static_cast<int>(S_tok), qkv_row_stride, BN)) return st;
 
@@ -916,6 +1242,8 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
   p.ws_part = split ? reinterpret_cast<float*>(static_cast<char*>(d_workspace) + kCountBytes)
                     : nullptr;
   p.block_mask = d_block_mask;
+  p.lpt_order = nullptr;
+  p.lpt_group = 0;
   p.o_row_stride = o_row_stride;
   p.F = F;
   p.N = N;
@@ -925,11 +1253,31 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
   p.nkv = static_cast<int>((S_tok + BN - 1) / BN);
   p.scale_log2 = static_cast<float>(static_cast<double>(softmax_scale) * 1.4426950408889634);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (d_block_mask)
-    return d == 128 ? launch<128, true>(mq, mk, mv, p, grid, di, s)
-                    : launch<64, true>(mq, mk, mv, p, grid, di, s);
-  return d == 128 ? launch<128, false>(mq, mk, mv, p, grid, di, s)
-                  : launch<64, false>(mq, mk, mv, p, grid, di, s);
+  if (d_block_mask) {
+    // With a workspace: costs and the longest-first order of the items in its partial-row
+    // area (unused by block-masked launches, which never split), when it holds them.
+    // Heads per ordered group: as many as fit their K/V in L2, and at least enough for four
+    // items per CTA.
+    const int64_t max_pairs = (tiles + 1) / 2;
+    const int64_t kv_head = 4 * S_tok * d;  // bytes of one head's K and V
+    int64_t g = di.l2_bytes / kv_head;
+    g = std::max<int64_t>(g, (4 * grid + max_pairs - 1) / max_pairs);
+    g = std::min<int64_t>(g, H);
+    if (split && g >= 1 && 2 * max_items * 4 <= workspace_bytes(d, grid) - kCountBytes) {
+      int* cost = reinterpret_cast<int*>(p.ws_part);
+      int* order = cost + max_items;
+      p.lpt_group = static_cast<int>(g);
+      item_cost_kernel<<<static_cast<unsigned>((max_items + 7) / 8), 256, 0, s>>>(p, cost);
+      if (rf_status st = launch_status("item_cost_kernel launch")) return st;
+      lpt_order_kernel<<<static_cast<unsigned>((H + g - 1) / g), 1024, 0, s>>>(p, cost, order);
+      if (rf_status st = launch_status("lpt_order_kernel launch")) return st;
+      p.lpt_order = order;
+    }
+    return d == 128 ? launch<128, true>(mq, mq128, mk, mv, p, grid, di, s)
+                    : launch<64, true>(mq, mq128, mk, mv, p, grid, di, s);
+  }
+  return d == 128 ? launch<128, false>(mq, mq128, mk, mv, p, grid, di, s)
+                  : launch<64, false>(mq, mq128, mk, mv, p, grid, di, s);
 }
 }  // namespace
 

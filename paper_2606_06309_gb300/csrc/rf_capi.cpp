@@ -37,7 +37,8 @@ rf_status current_device_info(DeviceInfo* out) {
         cudaDeviceGetAttribute(&n.cc_minor, cudaDevAttrComputeCapabilityMinor, dev) !=
             cudaSuccess ||
         cudaDeviceGetAttribute(&n.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
-            cudaSuccess)
+            cudaSuccess ||
+        cudaDeviceGetAttribute(&n.l2_bytes, cudaDevAttrL2CacheSize, dev) != cudaSuccess)
       return fail(RF_ERR_CUDA, "cudaDeviceGetAttribute", cudaGetLastError());
     d = n;
   }

@@ -14,6 +14,7 @@ struct DeviceInfo {
   int cc_major = 0;
   int cc_minor = 0;
   int max_smem_optin = 0;
+  int l2_bytes = 0;
 };
 
 // Properties of the current device, cached per device ordinal (thread-safe).

@@ -106,6 +106,11 @@ def test_device_calls_reject_bad_args_on_host(rf):
     args[14], args[15] = P, -1
     assert lib.rf_attn(*args) == 1                                   # negative workspace size
     assert lib.rf_attn_workspace_bytes(96) == -1
+    margs = [P, None, P, P, P, 256, 256, 4, 64, 2, 128, P, P, 0.1, None, None, 0, None, None]
+    assert lib.rf_attn_block_masked(*margs) == 1                      # null block mask
+    margs[14] = P
+    margs[7], margs[8] = 4097, 128
+    assert lib.rf_attn_block_masked(*margs) == 2                      # 4097 key blocks
 
 
 def _scene_proxies(F=21, E=960, starts=(0, 4, 9, 13, 17), noise=0.3, seed=0):

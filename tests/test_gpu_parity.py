@@ -554,6 +554,8 @@ def test_graph_replay_matches_eager(cuda_lib, name):
 # rf_attn_block_masked: frame mask x token block mask (Appendix D)
 # ---------------------------------------------------------------------------
 def _run_masked(rf, Q, K, V, F, N, mask, scale, bmask, split=True):
+    """split=True passes a workspace.  Block-masked launches never split; with a workspace
+    they take work items from a queue in its counter words and leave them at zero."""
     H, d = Q.shape[1], Q.shape[2]
     S_tok = F * N
     O = torch.full((S_tok, H, d), SENTINEL, dtype=torch.bfloat16, device=DEV)
@@ -638,3 +640,40 @@ def test_attn_block_masked_local_window_and_empty_items(cuda_lib):
         _check_masked(Q, K, V, O, L, mask, N, 1 / math.sqrt(d), bm, f"window split={split}")
         rows = _active_rows(mask, N)
         assert (O[rows, 1].float() == 0).all() and torch.isneginf(L[1, rows]).all()
+
+
+def test_attn_block_masked_more_than_1024_key_blocks(cuda_lib):
+    """1025 key blocks: a work item's tile bitmap runs past the first 1024 tiles, and one query
+    block may attend only to key blocks near the end (the last one ragged, 64 keys)."""
+    rf = cuda_lib
+    F, N, H, d = 2, 65600, 1, 64
+    Q, K, V = _qkv(F * N, H, d, seed=11)
+    nb = (F * N + 127) // 128
+    assert nb == 1025
+    rng = np.random.default_rng(3)
+    bm = (rng.random((H, nb, nb)) < 0.02).astype(np.uint8)
+    bm[0, :, nb - 1] = 1
+    bm[0, 7, :] = 0
+    bm[0, 7, 1000:] = 1
+    scale = 1.0 / math.sqrt(d)
+    O, L = _run_masked(rf, Q, K, V, F, N, [1, 0], scale, bm, split=False)
+    rows = np.array([0, 1, 127, 7 * 128, 7 * 128 + 77, 8 * 128 - 1, 30000, 65599])
+    Oref, Lref = oracle.attention_block_masked(Q.cpu(), K.cpu(), V.cpu(), rows, scale, bm)
+    compare(O.cpu().float()[rows].numpy(), Oref, L.cpu()[:, rows].numpy(), Lref,
+            "1025 key blocks")
+
+
+@pytest.mark.parametrize("split", [True, False])
+def test_attn_block_masked_causal_blocks(cuda_lib, split):
+    """A causal block mask (key block <= query block): work items differ in cost from one
+    key tile to all of them, which the longest-first work queue (with a workspace) and the
+    round-robin deal (without) must both compute exactly."""
+    rf = cuda_lib
+    F, N, H, d = 4, 512, 3, 128
+    Q, K, V = _qkv(F * N, H, d, seed=23)
+    nb = (F * N + 127) // 128
+    qb, kb = np.meshgrid(np.arange(nb), np.arange(nb), indexing="ij")
+    bm = np.broadcast_to((kb <= qb).astype(np.uint8), (H, nb, nb)).copy()
+    mask = [1, 1, 0, 1]
+    O, L = _run_masked(rf, Q, K, V, F, N, mask, 1 / math.sqrt(d), bm, split)
+    _check_masked(Q, K, V, O, L, mask, N, 1 / math.sqrt(d), bm, f"causal split={split}")
