@@ -39,8 +39,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic of one rf_attn launch measured with ncu (dram__bytes_read.sum +
 # dram__bytes_write.sum; the capture is summarised in profiles/attn_kernel_small_all_active.md).
 # It is reported only while the kernel source still has this hash.
-ATTN_TRAFFIC = {"sha256_rf_attn_cu": "4e1962ceef5626c81f69fa626db9082fdc3dd03f44330f72797c3daafc7aa99b",
-                "workload": "small", "bytes_per_launch": 188480768 + 47935744,
+ATTN_TRAFFIC = {"sha256_rf_attn_cu": "5a1a0e5a60c77656d68521e8384b5963909b43d9fe38c5ec450be09d4813b15d",
+                "workload": "small", "bytes_per_launch": 187772160 + 46801152,
                 "launch": "schedule step 0 of the small workload (all 13 frames active)"}
 
 
