@@ -336,11 +336,14 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
     ms, flops, _ = combine_ranks(t0.elapsed_time(t1),
                                  float(sum(flops_step[k % S] for k in range(K_steps))), dist,
                                  Q.device)
-    h2d, d2h = pipe.bytes_per_step()
+    h2d, d2h = pipe.bytes_per_step(last=K_steps)
     return {"value": round(flops / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "steps": K_steps,
             "ms_per_step": round(ms / K_steps, 5), "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h,
-            "overlap": "H2D of step k+1 and D2H of step k-1 overlap the compute of step k"}
+            "overlap": "three buffer sets: H2D of steps k+1, k+2 and D2H of earlier steps "
+                       "overlap the compute of step k",
+            "copied": "in: active frames' Q rows, all of K and V, the velocity; out: active "
+                      "frames' O rows, the latent store (bytes averaged over the timed steps)"}
 
 
 def run_bandwidth(w, dev, peaks):

@@ -385,6 +385,8 @@ def test_host_pipeline_matches_device_path(cuda_lib, name):
         act = np.array(_active_rows(oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)["mask"][s], w.N))
         assert torch.equal(hO[s][act], outs[s][0][act]), s
         assert torch.equal(hz[s], outs[s][1]), s
+        skipped = np.setdiff1d(np.arange(w.S_tok), act)
+        assert (hO[s][skipped] == 0).all(), s      # rows no step writes are not copied back
     assert core.status.item() == 0
 
 
