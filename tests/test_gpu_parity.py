@@ -255,7 +255,8 @@ def test_attn_planted_keys(cuda_lib):
     assert err < 2e-2, err
 
 
-@pytest.mark.parametrize("name,steps", [("small", (0, 1)), ("large", (0, 1))])
+@pytest.mark.parametrize("name,steps", [("small", (0, 1)), ("mid", (0, 18)), ("large", (0, 1)),
+                                        ("long", (0, 12))])
 def test_attn_full_size_sampled_rows(cuda_lib, name, steps):
     """The benchmark's launch configuration at full size; sampled rows against
     the oracle: the first and last row of every active frame, the rows around
