@@ -108,7 +108,8 @@ struct AttnParams {
   float* ws_part;  // [kMaxGrid][2][BM][D+4] partial rows
   const uint8_t* block_mask;  // [H][nkv][nkv] token block mask (128-token blocks), or null
   const int* lpt_order;       // (block mask, with a workspace) unit order for the queue, or null
-  int lpt_group;              // heads per group of that order
+  int lpt_heads_l2;           // heads whose K/V fit in half of L2 (at least 1)
+  int lpt_grid;               // CTAs of the attention launch
   int64_t o_row_stride;
   int F, N, Np, H, S_tok, nkv;
   float scale_log2;
@@ -528,7 +529,6 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     tc_fence_after();
     return ok;
   };
-  const int nw = (p.nkv + 31) >> 5;
   for (int k = 0;; ++k) {  // k: units so far (MASKED: tile-list ring position)
     int w;
     const uint32_t* tw = nullptr;
@@ -543,9 +543,9 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     }
     const Unit u = get_unit(sc, p, w);
     const bool hasB = 2 * u.pr + 1 < sc.tiles;
-    // KV tiles of the unit: all of [j0, j1), or (MASKED) the bits of the builder's bitmap
-    int jc = u.j0;
-    if constexpr (MASKED) jc = next_kept(tw, 0, nw);
+    // number of KV tiles of the unit: j1 - j0, or (MASKED) the set bits of the builder's
+    // bitmap (the issuer needs only the count; the producer walks the bits)
+    const int ntiles = MASKED ? static_cast<int>(tw[kTLWords]) : u.j1 - u.j0;
     if (!mbar_wait(bar(C::kBarQFull + 0), q_cnt[0] & 1, abort, kWaitLimitNs)) goto fail;
     ++q_cnt[0];
     if (hasB) {
@@ -553,7 +553,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       ++q_cnt[1];
     }
     tc_fence_after();
-    if (MASKED && jc >= p.nkv) {
+    if (MASKED && ntiles == 0) {
       // no allowed key block: release the queries.  No output barrier is committed: the
       // softmax warps see the same empty tile list and write their result without waiting
       // (a commit here could run two phases ahead of them).
@@ -577,12 +577,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     int nj = 1;  // tiles issued so far
 #pragma unroll 1
     for (int j = 0;; ++j) {
-      if constexpr (MASKED) {
-        jc = next_kept(tw, jc + 1, nw);
-        if (jc >= p.nkv) break;
-      } else {
-        if (j + 1 >= u.j1 - u.j0) break;
-      }
+      if (j + 1 >= ntiles) break;
       ++nj;
       if (!next_slot(sK)) goto fail;
       mma_qk<D>(tS[0], dQ[0], dK(sK));
@@ -1008,69 +1003,132 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------------------------
-// Longest-first order of block-masked work items (two small launches before the attention
+// Longest-first order of block-masked work items (one small launch before the attention
 // kernel).  Under a mask, items differ in cost (the number of KV tiles their tile pair may
-// see); handing them out from the work queue longest first within each head (LPT list
-// scheduling) keeps the CTAs' finishing times close where a round-robin deal or the natural
-// order can leave costly items for the end (a causal block mask on 13 x 1560 tokens: 1.205 ms
-// dealt round-robin, 0.918 ms longest first).
-// ---------------------------------------------------------------------------------------
-// One warp per item: its cost is the number of set bits of the bitmap the builder will write.
-__global__ void __launch_bounds__(256) item_cost_kernel(const AttnParams p, int* cost) {
-  const Sched sc = make_sched(p);  // a block-masked launch: no split, so units are items
-  const int lane = threadIdx.x & 31;
-  const int item = blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (item >= sc.units) return;
-  const Unit u = get_unit(sc, p, item);
-  const QRanges q = unit_qranges(p, sc, u);
-  int total = 0;
-  for (int j0 = 0; j0 < p.nkv; j0 += 32) {
-    const int j = j0 + lane;
-    bool ok = false;
-    if (j < p.nkv)
-      for (int i = 0; i < q.n; ++i)
-        for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb)
-          ok = ok || q.mh[static_cast<int64_t>(qb) * p.nkv + j] != 0;
-    total += __popc(__ballot_sync(0xffffffffu, ok));
-  }
-  if (lane == 0) cost[item] = total;
+// see); handing them out from the work queue longest first within each group of heads (LPT
+// list scheduling) keeps the CTAs' finishing times close where a round-robin deal or the
+// natural order can leave costly items for the end (a causal block mask on 13 x 1560 tokens:
+// 1.10 ms dealt round-robin, 0.83 ms longest first).
+//
+// Groups of consecutive heads (item = head * pairs + pair): the queue hands out the groups one
+// after the other, so the CTAs that run together work on the heads of one group.  A group has
+// as many heads as fit their K/V in half of L2, and at least enough for six items per CTA
+// (from the active count, so on the device): one global order by cost spread the CTAs over
+// all 40 heads of a 21 x 3600-token workload (39 MB of K/V per head, 129 MB of L2) and was 5%
+// slower than no order at all, while one head per group left 13 x 1560 tokens (80 items per
+// head, 152 CTAs) 19% slower than the global order, because each head's costly items started
+// late.
+__device__ __forceinline__ int lpt_group_heads(const AttnParams& p, const Sched& sc) {
+  const int need = (6 * p.lpt_grid + sc.pairs - 1) / max(sc.pairs, 1);
+  return min(p.H, max(p.lpt_heads_l2, need));
 }
+//
+// Each CTA covers kPrepassItems items of one head, one warp per item: the item's cost is the
+// number of set bits of the bitmap the builder will write, found with each lane loading 32
+// independent mask bytes per query block.  The CTA that completes a group (a counter per group
+// in the workspace, reset by that CTA) sorts the group by decreasing cost with a counting sort.
+// The order among equal costs is arbitrary, which changes no result (every item is computed
+// the same way by whichever CTA takes it) and, within an L2-sized group, no locality.
+constexpr int kPrepassItems = 8;       // items (warps) per CTA
+constexpr int kPrepassThreads = 32 * kPrepassItems;
+constexpr int kQueueGroup0 = 2;        // first per-group counter word
+constexpr int kMaxLptGroups = kMaxGrid - kQueueGroup0;
+constexpr int kCostBins = kTLMaxTiles + 1;
+constexpr int kBinsPerThread = (kCostBins + kPrepassThreads - 1) / kPrepassThreads;
 
-// Groups of lpt_group consecutive heads: each group's items (item = head * pairs + pair) by
-// decreasing cost.  The queue hands out the groups one after the
-// other, so the CTAs that run together work on the heads of one group, whose K/V the host sized
-// to fit in L2: one global order by cost spread them over all 40 heads of a 21 x 3600-token
-// workload (39 MB of K/V per head, 129 MB of L2) and was 5% slower than no order at all.  The
-// host also makes a group hold several items per CTA, so that its costly items do not start
-// late: one head per group left 13 x 1560 tokens (80 items per head, 152 CTAs) 19% slower
-// than the global order.
-// The order is stable (equal costs keep item order, so CTAs taking items of equal cost still
-// walk the heads in turn; an unstable counting sort left the L2 hit rate at 81% instead of
-// 94% on the band mask of 13 x 1560 tokens): each thread ranks one item of its group,
-// rank(i) = #{j : c_j > c_i} + #{j < i : c_j = c_i}, against the group's costs in shared
-// memory.  A group of n items takes ceil(n / kOrderThreads) CTAs.
-constexpr int kOrderThreads = 128;
-constexpr int kLptMaxItems = 8192;  // items per group (32 KB of costs)
-__global__ void __launch_bounds__(kOrderThreads) lpt_order_kernel(const AttnParams p,
-                                                                  const int* cost, int* order,
-                                                                  int ctas_per_group) {
-  __shared__ int c[kLptMaxItems];
-  const Sched sc = make_sched(p);
-  const int group = blockIdx.x / ctas_per_group, part = blockIdx.x % ctas_per_group;
-  const int base = group * p.lpt_group * sc.pairs;
-  const int n = min(p.lpt_group * sc.pairs, sc.units - base);
-  if (n <= 0 || n > kLptMaxItems) return;  // the host keeps every group within kLptMaxItems
-  for (int i = threadIdx.x; i < n; i += blockDim.x) c[i] = cost[base + i];
-  __syncthreads();
-  const int i = part * kOrderThreads + threadIdx.x;
-  if (i >= n) return;
-  const int ci = c[i];
-  int r = 0;
-  for (int j = 0; j < n; ++j) {
-    const int cj = c[j];
-    r += (cj > ci) || (cj == ci && j < i);
+__global__ void __launch_bounds__(kPrepassThreads)
+    lpt_prepass_kernel(const AttnParams p, int* cost, int* order, int ctas_per_head) {
+  __shared__ int start[kBinsPerThread * kPrepassThreads];  // bin b holds cost kTLMaxTiles - b
+  __shared__ int warp_sum[kPrepassThreads / 32];
+  __shared__ int last;
+  const Sched sc = make_sched(p);  // a block-masked launch: no split, so units are items
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int h = blockIdx.x / ctas_per_head, part = blockIdx.x % ctas_per_head;
+  const int ctas_head = (sc.pairs + kPrepassItems - 1) / kPrepassItems;
+  if (sc.pairs == 0 || part >= ctas_head) return;  // CTA-uniform: no item of this head
+  const int gh = lpt_group_heads(p, sc);
+  const int group = h / gh;
+  const int base = group * gh * sc.pairs;                  // the group's first item
+  const int heads = min(gh, p.H - group * gh);
+  const int n = heads * sc.pairs;                          // the group's items
+  const int item = (h - group * gh) * sc.pairs + part * kPrepassItems + wid;  // in the group
+  if (part * kPrepassItems + wid < sc.pairs) {
+    const Unit u = get_unit(sc, p, base + item);
+    const QRanges q = unit_qranges(p, sc, u);
+    const int nw = (p.nkv + 31) >> 5;
+    int total = 0;
+    for (int k0 = 0; k0 < nw; k0 += 32) {
+      uint32_t acc = 0;  // bit l: tile (k0 + l) * 32 + lane allowed
+      for (int i = 0; i < q.n; ++i)
+        for (int qb = q.lo[i]; qb <= q.hi[i]; ++qb) {
+          const uint8_t* mrow = q.mh + static_cast<int64_t>(qb) * p.nkv;
+#pragma unroll
+          for (int l = 0; l < 32; ++l) {
+            const int j = (k0 + l) * 32 + lane;
+            if (j < p.nkv && mrow[j] != 0) acc |= 1u << l;
+          }
+        }
+      total += __popc(acc);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) total += __shfl_xor_sync(0xffffffffu, total, off);
+    if (lane == 0) {
+      cost[base + item] = total;
+      __threadfence();  // visible to the CTA that sorts the group
+    }
   }
-  order[base + r] = base + i;
+  // the CTA that completes the group sorts it
+  const int ctas = heads * ctas_head;
+  __syncthreads();
+  if (tid == 0) {
+    int* counter = p.ws_count + kQueueGroup0 + group;
+    last = atomicAdd(counter, 1) == ctas - 1;
+    if (last) *counter = 0;  // ready for the next launch
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  for (int i = tid; i < kBinsPerThread * kPrepassThreads; i += kPrepassThreads) start[i] = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += kPrepassThreads)
+    atomicAdd(&start[kTLMaxTiles - __ldcg(cost + base + i)], 1);
+  __syncthreads();
+  // exclusive prefix sum over the bins: kBinsPerThread consecutive bins per thread, then a
+  // block-wide scan of the per-thread sums
+  int own[kBinsPerThread];
+  int sum = 0;
+#pragma unroll
+  for (int b = 0; b < kBinsPerThread; ++b) {
+    own[b] = start[tid * kBinsPerThread + b];
+    sum += own[b];
+  }
+  int incl = sum;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += t;
+  }
+  if (lane == 31) warp_sum[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    int v = lane < kPrepassThreads / 32 ? warp_sum[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, v, off);
+      if (lane >= off) v += t;
+    }
+    if (lane < kPrepassThreads / 32) warp_sum[lane] = v;  // inclusive, over warps
+  }
+  __syncthreads();
+  int run = incl - sum + (wid > 0 ? warp_sum[wid - 1] : 0);
+#pragma unroll
+  for (int b = 0; b < kBinsPerThread; ++b) {
+    start[tid * kBinsPerThread + b] = run;
+    run += own[b];
+  }
+  __syncthreads();
+  for (int i = tid; i < n; i += kPrepassThreads)
+    order[base + atomicAdd(&start[kTLMaxTiles - __ldcg(cost + base + i)], 1)] = base + i;
 }
 
 // ---------------------------------------------------------------------------------------
@@ -1216,7 +1274,8 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
                     : nullptr;
   p.block_mask = d_block_mask;
   p.lpt_order = nullptr;
-  p.lpt_group = 0;
+  p.lpt_heads_l2 = 1;
+  p.lpt_grid = 0;
   p.o_row_stride = o_row_stride;
   p.F = F;
   p.N = N;
@@ -1229,23 +1288,20 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
   if (d_block_mask) {
     // With a workspace: costs and the longest-first order of the items in its partial-row
     // area (unused by block-masked launches, which never split), when it holds them.
-    // Heads per ordered group: as many as fit their K/V in L2, and at least enough for four
-    // items per CTA; at most kLptMaxItems items.
+    // Heads whose K/V fit in half of L2; the kernel makes groups of at least that many heads.
     const int64_t max_pairs = (tiles + 1) / 2;
     const int64_t kv_head = 4 * S_tok * d;  // bytes of one head's K and V
-    int64_t g = di.l2_bytes / kv_head;
-    g = std::max<int64_t>(g, (4 * grid + max_pairs - 1) / max_pairs);
-    g = std::min<int64_t>({g, H, kLptMaxItems / max_pairs});
-    if (split && g >= 1 && 2 * max_items * 4 <= workspace_bytes(d, grid) - kCountBytes) {
+    const int64_t heads_l2 = std::max<int64_t>(1, di.l2_bytes / 2 / kv_head);
+    if (split && (H + heads_l2 - 1) / heads_l2 <= kMaxLptGroups &&
+        2 * max_items * 4 <= workspace_bytes(d, grid) - kCountBytes) {
       int* cost = reinterpret_cast<int*>(p.ws_part);
       int* order = cost + max_items;
-      p.lpt_group = static_cast<int>(g);
-      item_cost_kernel<<<static_cast<unsigned>((max_items + 7) / 8), 256, 0, s>>>(p, cost);
-      if (rf_status st = launch_status("item_cost_kernel launch")) return st;
-      const int per_group = static_cast<int>((g * max_pairs + kOrderThreads - 1) / kOrderThreads);
-      lpt_order_kernel<<<static_cast<unsigned>((H + g - 1) / g * per_group), kOrderThreads, 0, s>>>(
-          p, cost, order, per_group);
-      if (rf_status st = launch_status("lpt_order_kernel launch")) return st;
+      p.lpt_heads_l2 = static_cast<int>(std::min<int64_t>(heads_l2, H));
+      p.lpt_grid = grid;
+      const int per_head = static_cast<int>((max_pairs + kPrepassItems - 1) / kPrepassItems);
+      lpt_prepass_kernel<<<static_cast<unsigned>(H * per_head), kPrepassThreads, 0, s>>>(
+          p, cost, order, per_head);
+      if (rf_status st = launch_status("lpt_prepass_kernel launch")) return st;
       p.lpt_order = order;
     }
     return d == 128 ? launch<128, true>(mq, mq128, mk, mv, p, grid, di, s)
