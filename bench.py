@@ -39,8 +39,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic of one rf_attn launch measured with ncu (dram__bytes_read.sum +
 # dram__bytes_write.sum; the capture is summarised in profiles/attn_kernel_small_all_active.md).
 # It is reported only while the kernel source still has this hash.
-ATTN_TRAFFIC = {"sha256_rf_attn_cu": "5a1a0e5a60c77656d68521e8384b5963909b43d9fe38c5ec450be09d4813b15d",
-                "workload": "small", "bytes_per_launch": 187772160 + 46801152,
+ATTN_TRAFFIC = {"sha256_rf_attn_cu": "57603a16f25ecdbbe6317a2af4577134ed9432cb2fef042d00c2223cc894ce6c",
+                "workload": "small", "bytes_per_launch": 187693568 + 46976768,
                 "launch": "schedule step 0 of the small workload (all 13 frames active)"}
 
 
