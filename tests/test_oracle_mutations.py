@@ -40,13 +40,15 @@ PIN_CALLS = [
     (pins.test_keyframes_threshold_direction, {}),
     (pins.test_kv_cache_endpoints_and_store, {}),
     (pins.test_kv_cache_commutes_with_affine_map, {}),
+    (pins.test_block_masked_attention_matches_sdpa_with_mask, {}),
+    (pins.test_block_masked_attention_all_allowed_is_dense_and_empty_rows_zero, {}),
 ]
 
 
 # the unmutated functions, captured before any test patches the module
 ORIG = {name: getattr(ro, name) for name in
         ("project", "euler", "attention", "schedule", "compact", "keyframe_select",
-         "project_kv_cache")}
+         "project_kv_cache", "attention_block_masked")}
 
 
 def _failures():
@@ -135,6 +137,11 @@ def _kv_slots_swapped(KV, cache, cur_slot, alpha, mask):
     return ORIG['project_kv_cache'](KV, cache, 1 - np.asarray(cur_slot), alpha, mask)
 
 
+def _block_mask_transposed(Q, K, V, rows, scale, block_mask, block=128, heads=None):
+    bm = np.swapaxes(np.asarray(block_mask), 1, 2)                   # [h][kb][qb]
+    return ORIG['attention_block_masked'](Q, K, V, rows, scale, bm, block, heads)
+
+
 MUTANTS = {
     "project: weights swapped": ("project", _project_swapped),
     "project: (1 - alpha) dropped": ("project", _project_dropped),
@@ -149,6 +156,7 @@ MUTANTS = {
     "compact: token index off by one": ("compact", _compact_token_shift),
     "keyframe_select: threshold step direction": ("keyframe_select", _keyframe_direction),
     "project_kv_cache: slots exchanged": ("project_kv_cache", _kv_slots_swapped),
+    "attention_block_masked: mask transposed": ("attention_block_masked", _block_mask_transposed),
 }
 
 
