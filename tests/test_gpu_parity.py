@@ -680,3 +680,18 @@ def test_attn_block_masked_causal_blocks(cuda_lib, split):
     mask = [1, 1, 0, 1]
     O, L = _run_masked(rf, Q, K, V, F, N, mask, 1 / math.sqrt(d), bm, split)
     _check_masked(Q, K, V, O, L, mask, N, 1 / math.sqrt(d), bm, f"causal split={split}")
+
+
+@pytest.mark.parametrize("split", [True, False])
+def test_attn_block_masked_empty_active_set(cuda_lib, split):
+    """No active frame: nothing is written, the status stays clear and (with a workspace) the
+    work-queue words are back at zero, so the next call on the same workspace is correct."""
+    rf = cuda_lib
+    F, N, H, d = 3, 512, 2, 128
+    Q, K, V = _qkv(F * N, H, d, seed=31)
+    nb = (F * N + 127) // 128
+    bm = np.ones((H, nb, nb), np.uint8)
+    O, L = _run_masked(rf, Q, K, V, F, N, [0, 0, 0], 1 / math.sqrt(d), bm, split)
+    assert (O.float() == SENTINEL).all() and (L == SENTINEL).all()
+    O, L = _run_masked(rf, Q, K, V, F, N, [0, 1, 0], 1 / math.sqrt(d), bm, split)
+    _check_masked(Q, K, V, O, L, [0, 1, 0], N, 1 / math.sqrt(d), bm, f"after empty split={split}")
