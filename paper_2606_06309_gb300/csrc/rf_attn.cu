@@ -10,9 +10,9 @@
 //               when the tile lies in one active frame, else gathered by frame index in
 //               8-row boxes) and streams K/V tiles of 128 tokens through a ring of
 //               shared-memory slots.
-//   warp 2      (block-masked launches) builds each work item's list of KV tiles.
 //   warp 1      owns TMEM (512 columns) and one lane issues every tcgen05.mma:
 //               S = Q K^T (both operands in shared memory) and O += P V (P in TMEM).
+//   warp 2      (block-masked launches) builds each work item's list of KV tiles.
 //   warps 4-7   softmax for query tile A, warps 8-11 for query tile B: thread = query row;
 //               online softmax in fp32 with base-2 exponentials, lazy rescaling of the O
 //               accumulator (only when the running max grows by more than 2^8), P rounded
@@ -30,11 +30,13 @@
 //
 // Work item = (head, pair of 128-row query tiles) over the flattened list of active rows
 // (each frame padded to a multiple of 8 rows); items are dealt round-robin to the CTAs, so
-// consecutive CTAs share the same head's K/V through L2.  When the last round of items would
-// leave more than half of the CTAs idle and the caller supplied a workspace, each item of that
-// round is split into C ranges of KV tiles (split-KV): every range writes its unnormalised
-// O row, running max and sum to the workspace, and the CTA that finishes the last range of an
-// item merges them (counter per item and query tile, reset to zero by the merging CTA).
+// consecutive CTAs share the same head's K/V through L2 (block-masked launches with a
+// workspace take items from a longest-first work queue instead).  When the last round of items
+// would leave more than half of the CTAs idle and the caller supplied a workspace, each item of
+// that round is split into C ranges of KV tiles (split-KV, unmasked launches only): every range
+// writes its unnormalised O row, running max and sum to the workspace, and the CTA that
+// finishes the last range of an item merges them (counter per item and query tile, reset to
+// zero by the merging CTA).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -305,9 +307,10 @@ constexpr int kQueueNext = 0, kQueueDone = 1;
 // ---------------------------------------------------------------------------------------
 // For every unit of this CTA, in order, one ring slot receives the bitmap of the KV tiles the
 // unit visits: the tiles some query block of its rows may attend to (block-masked launches
-// never split, so a unit is a whole item).  The other roles walk this bitmap, so the block
-// mask in global memory is scanned once per unit, with 32 lanes loading independent bytes,
-// instead of tile by tile on the critical paths of the producer and the MMA issuer.
+// never split, so a unit is a whole item).  The producer and the softmax warps walk this
+// bitmap and the MMA issuer uses its count, so the block mask in global memory is scanned once
+// per unit, with 32 lanes loading independent bytes, instead of tile by tile on the critical
+// paths of the producer and the MMA issuer.
 __device__ __forceinline__ void tile_list_builder(const AttnParams& p, const Sched& sc,
                                                   const TLRing& tl, volatile int* abort) {
   const int lane = threadIdx.x & 31;
@@ -1170,7 +1173,10 @@ rf_status make_map(CUtensorMap* m, const void* base, int d, int H, int S_tok, in
   return RF_OK;
 }
 
-// Workspace layout: [kMaxGrid] int merge counters, then (256-byte aligned) the partial rows.
+// Workspace layout: [kMaxGrid] int counters, then (256-byte aligned) the partial rows.
+// Unmasked launches use the counters to merge split-KV ranges and the rest for the partials.
+// Block-masked launches (which never split) use counters 0 and 1 for the work queue, 2.. for
+// the longest-first pre-pass's groups, and the partial-row area for the items' costs and order.
 constexpr int64_t kCountBytes = kMaxGrid * 4;
 int64_t workspace_bytes(int d, int grid) {
   return kCountBytes + static_cast<int64_t>(grid) * 2 * BM * (d + 4) * 4;
