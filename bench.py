@@ -549,6 +549,24 @@ def run_sweep(w, dev, Q, K, V, O, vel, steps):
 # ---------------------------------------------------------------------------
 # CPU oracle (baseline leg and the reference arm)
 # ---------------------------------------------------------------------------
+def _cpu_model():
+    """The host CPU as /proc/cpuinfo names it (on aarch64: implementer and part codes)."""
+    info = {}
+    try:
+        for line in open("/proc/cpuinfo", encoding="utf-8"):
+            k, _, v = line.partition(":")
+            k = k.strip().lower()
+            if k in ("model name", "cpu implementer", "cpu part") and k not in info:
+                info[k] = v.strip()
+    except OSError:
+        pass
+    import platform
+    if "model name" in info:
+        return info["model name"]
+    parts = [f"{k} {info[k]}" for k in ("cpu implementer", "cpu part") if k in info]
+    return platform.machine() + (" (" + ", ".join(parts) + ")" if parts else "")
+
+
 def cpu_baseline(w, budget_s=15.0):
     """The fp64 oracle as it stands, on a bounded sample of one step: schedule,
     projection and Euler update for every frame at latent width, and attention for a
@@ -581,7 +599,7 @@ def cpu_baseline(w, budget_s=15.0):
             break
         n *= 2
     return {"value": round(flops / elapsed / 1e12, 6), "unit": UNIT, "cores": os.cpu_count(),
-            "kind": "oracle", "seconds": round(elapsed, 2),
+            "cpu": _cpu_model(), "kind": "oracle", "seconds": round(elapsed, 2),
             "sample": f"step {s} of {w.name}: full schedule/projection/Euler at latent width "
                       f"plus attention of sampled active rows x {w.H} heads x {w.S_tok} keys "
                       f"(fp64 numpy, {flops / 1e12:.3f} TFLOP)"}
@@ -608,7 +626,7 @@ def run_reference(args):
            "config": {"workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads "
                                   f"x {w.d}, latent {w.C} ch, {w.S} flow-matching steps"},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
-                            "kind": "oracle", "sample": vals[0]["sample"]},
+                            "cpu": vals[0]["cpu"], "kind": "oracle", "sample": vals[0]["sample"]},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
