@@ -15,9 +15,10 @@ from typing import Optional
 import numpy as np
 
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
-           "rf_project", "rf_project_kv", "rf_attn", "rf_attn_block_masked", "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step",
-           "rf_frame_gram", "rf_keyframe_select", "rf_status_str",
-           "rf_version", "EXPORTS"]
+           "rf_project", "rf_project_kv", "rf_attn", "rf_attn_block_masked",
+           "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step", "rf_frame_gram",
+           "rf_keyframe_select", "rf_selftest_bounded_wait", "rf_status_str", "rf_version",
+           "EXPORTS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB: Optional[ctypes.CDLL] = None
