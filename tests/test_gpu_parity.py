@@ -695,3 +695,79 @@ def test_attn_block_masked_empty_active_set(cuda_lib, split):
     assert (O.float() == SENTINEL).all() and (L == SENTINEL).all()
     O, L = _run_masked(rf, Q, K, V, F, N, [0, 1, 0], 1 / math.sqrt(d), bm, split)
     _check_masked(Q, K, V, O, L, [0, 1, 0], N, 1 / math.sqrt(d), bm, f"after empty split={split}")
+
+
+# ---------------------------------------------------------------------------
+# Bandwidth kernels at the hidden-width stress shape the bench times (C = H*d), sampled
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,s", [("small", 1), ("large", 14)])
+def test_bandwidth_kernels_at_stress_shape_sampled(cuda_lib, name, s):
+    """rf_project, rf_step and rf_project_kv on the full hidden-width buffers of the workload
+    (up to 1.5 GB per fp32 buffer), at a step with skipped frames; 65536 sampled elements per
+    frame against the oracle, which computes them one by one."""
+    rf = cuda_lib
+    w = wl.get(name)
+    D = w.H * w.d
+    E = w.N * D
+    p = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+    mask = p["mask"][s].astype(np.uint8)
+    assert 0 < mask.sum() < w.F
+    slot = p["cur_slot"][s].astype(np.uint8)
+    alpha = p["alpha"][s].astype(np.float32)
+    beta = (1.0 - p["alpha"][s]).astype(np.float32)
+    dt = p["dt"][s].astype(np.float32)
+    g = torch.Generator(device=DEV).manual_seed(7 + s)
+    z2 = torch.randn(2, w.F, E, generator=g, device=DEV)
+    v = torch.randn(w.F, E, generator=g, device=DEV)
+    act = torch.zeros(w.F, dtype=torch.int32, device=DEV)
+    skp = torch.zeros(w.F, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(torch.from_numpy(mask).to(DEV), w.F, w.N, act, skp, None, cnt)
+    rng = np.random.default_rng(s)
+    idx = torch.from_numpy(np.sort(rng.choice(E, size=65536, replace=False))).to(DEV)
+    frames = torch.arange(w.F, device=DEV)
+    sl = torch.from_numpy(slot.astype(np.int64)).to(DEV)
+    cur = z2[sl, frames][:, idx].cpu().double().numpy()
+    prev = z2[1 - sl, frames][:, idx].cpu().double().numpy()
+    # Eq. 3 projection
+    ctx = torch.full((w.F, E), SENTINEL, device=DEV)
+    rf.rf_project(ctx, z2, torch.from_numpy(slot).to(DEV), torch.from_numpy(alpha).to(DEV),
+                  torch.from_numpy(beta).to(DEV), w.F, E)
+    got = ctx[:, idx].cpu().double().numpy()
+    want = oracle.project(prev, cur, p["alpha"][s])
+    terms = np.abs(beta.astype(np.float64))[:, None] * np.abs(prev) + \
+        np.abs(alpha.astype(np.float64))[:, None] * np.abs(cur)
+    assert _rel_err(got, want, terms) <= 1e-5
+    del ctx
+    # Euler update of the active frames into the other slot
+    vs = v[:, idx].cpu().double().numpy()
+    rf.rf_step(z2, torch.from_numpy(slot).to(DEV), v, torch.from_numpy(dt).to(DEV), act, cnt,
+               w.F, E)
+    got_new = z2[1 - sl, frames][:, idx].cpu().double().numpy()
+    m = mask.astype(bool)
+    want = oracle.euler(cur, vs, dt.astype(np.float64))
+    terms = np.abs(cur) + np.abs(dt.astype(np.float64))[:, None] * np.abs(vs)
+    assert _rel_err(got_new[m], want[m], terms[m]) <= 1e-5
+    np.testing.assert_array_equal(got_new[~m], prev[~m])       # skipped frames untouched
+    del z2, v
+    # rolling K/V cache: projected rows of skipped frames, fresh rows stored for active ones
+    K = torch.randn(w.F * w.N, D, generator=g, device=DEV).to(torch.bfloat16)
+    Kc = torch.randn(2, w.F, w.N, D, generator=g, device=DEV).to(torch.bfloat16)
+    Vv = torch.randn(w.F * w.N, D, generator=g, device=DEV).to(torch.bfloat16)
+    Vc = torch.randn(2, w.F, w.N, D, generator=g, device=DEV).to(torch.bfloat16)
+    kcur = Kc[sl, frames].reshape(w.F, E)[:, idx].cpu().double().numpy()
+    kprev = Kc[1 - sl, frames].reshape(w.F, E)[:, idx].cpu().double().numpy()
+    kfresh = K.view(w.F, E)[:, idx].cpu().double().numpy()
+    rf.rf_project_kv(K, Vv, K.stride(0), Kc, Vc, torch.from_numpy(slot).to(DEV),
+                     torch.from_numpy(alpha).to(DEV), torch.from_numpy(beta).to(DEV), act, skp,
+                     cnt, w.F, w.N, D)
+    got_k = K.view(w.F, E)[:, idx].cpu().double().numpy()
+    want_k = oracle.project(kprev, kcur, p["alpha"][s])
+    terms = np.abs(beta.astype(np.float64))[:, None] * np.abs(kprev) + \
+        np.abs(alpha.astype(np.float64))[:, None] * np.abs(kcur)
+    sk = ~m
+    assert (np.abs(got_k[sk] - want_k[sk]) <= 2.0 ** -8 * terms[sk] + 1e-30).all()
+    np.testing.assert_array_equal(got_k[m], kfresh[m])          # active rows untouched
+    stored = Kc[1 - sl, frames].reshape(w.F, E)[:, idx].cpu().double().numpy()
+    np.testing.assert_array_equal(stored[m], kfresh[m])         # fresh rows shifted in
+    np.testing.assert_array_equal(stored[sk], kprev[sk])        # skipped frames' cache kept
