@@ -210,6 +210,10 @@ def test_attn_tiny_every_step(cuda_lib):
     (2, 8, 2, 64, [1, 1]),                # one tile, no second tile
     (7, 136, 2, 128, [1, 1, 1, 0, 1, 1, 1]),
     (1, 130, 1, 64, [1]),                 # KV tail of 2 keys
+    (40, 8, 2, 64, [1, 0] * 20),          # a 128-row tile spans 16 frames (8-row gather)
+    (64, 1, 2, 128, [1, 1, 0, 1] * 16),   # N = 1: seven padded rows per frame
+    (3, 4096, 1, 128, [1, 0, 1]),         # frames of whole tiles (one 128-row box each)
+    (2, 1, 1, 64, [1, 1]),                # two tokens in all
 ])
 def test_attn_ragged_shapes(cuda_lib, F, N, H, d, mask):
     rf = cuda_lib
