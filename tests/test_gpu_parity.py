@@ -607,6 +607,9 @@ def _check_masked(Q, K, V, O, L, mask, N, scale, bmask, label):
     (5, 100, 2, 64, [1, 0, 1, 1, 0], 0.6, True),     # N % 8 != 0
     (3, 1560, 2, 128, [1, 0, 1], 0.4, True),         # ragged KV tail, several tiles per frame
     (3, 1560, 2, 128, [1, 1, 1], 0.15, False),
+    # 8-token frames, every 32nd active: a tile pair holds 32 frames in 32 separate query
+    # blocks, more ranges than a unit keeps, so the last range is widened (a superset)
+    (1024, 8, 2, 64, ([1] + [0] * 31) * 32, 0.3, True),
 ])
 def test_attn_block_masked_parity(cuda_lib, F, N, H, d, mask, density, split):
     rf = cuda_lib
