@@ -207,10 +207,12 @@ rf_status rf_attn(void* d_O, float* d_lse, const void* d_Q, const void* d_K, con
  * work item may attend to are not loaded or multiplied at all.  A row that may attend to
  * no key gets O = 0 and LSE = -inf.  All other arguments, requirements and results are
  * those of rf_attn, except for the workspace: the work is never split into KV ranges, and
- * with a workspace (same size and rules as for rf_attn) the CTAs take work items from a
- * queue kept in its first two counter words, which the kernel leaves at zero; without one,
- * items are dealt round-robin.  Returns RF_ERR_INVALID_ARG for a null mask and
- * RF_ERR_UNSUPPORTED for more than 4096 key blocks (F*N > 524288 tokens).
+ * with a workspace (same size and rules as for rf_attn) a small pre-pass launch orders the
+ * work items longest first within groups of heads and the CTAs take them from a queue.  The
+ * queue and the groups use the workspace's counter words, which the calls leave at zero, and
+ * the items' costs and order use its partial-row area.  Without a workspace, items are dealt
+ * round-robin.  Returns RF_ERR_INVALID_ARG for a null mask and RF_ERR_UNSUPPORTED for more
+ * than 4096 key blocks (F*N > 524288 tokens).
  */
 rf_status rf_attn_block_masked(void* d_O, float* d_lse, const void* d_Q, const void* d_K,
                                const void* d_V, int64_t qkv_row_stride, int64_t o_row_stride,
