@@ -238,6 +238,20 @@ def run_gpu(args):
     per_launch_flops = attn_flops_total / len(ev)
     # all-frames-active comparison, same number of steps
     ms_all, _ = timed(core_all, K_steps, min(W_steps, 3))
+    # per schedule step: attention launch time against the all-active launch
+    _, ev_all = timed(core_all, S, 3, per_launch=True)
+    attn_all_ms = statistics.mean(a.elapsed_time(b) for _, a, b in ev_all)
+    by_step = {}
+    for (s_, _, _), t in zip(ev, launch_ms):
+        by_step.setdefault(s_, []).append(t)
+    per_step_ms = [statistics.mean(by_step[s_]) if s_ in by_step else None for s_ in range(S)]
+    per_step = {
+        "attn_ms": [round(t, 5) if t is not None else None for t in per_step_ms],
+        "attn_ms_all_active": round(attn_all_ms, 5),
+        "attn_speedup": [round(attn_all_ms / t, 3) if t else None for t in per_step_ms],
+        "ideal_attn_speedup": [round(w.F / int(A_per_step[s_]), 3) if A_per_step[s_] else None
+                               for s_ in range(S)],
+    }
     # the same trajectory replayed from one CUDA graph (launch overhead removed)
     graph_ms = None
     try:
@@ -290,6 +304,7 @@ def run_gpu(args):
         "speedup_vs_all_active": round(ms_all / ms, 4),
         "ideal_speedup_vs_all_active": round(K_steps * flops_all /
                                              sum(flops_step[k % S] for k in range(K_steps)), 4),
+        "per_step": per_step,
         "roofline": {
             "bound": "tensor", "kernel": "rf_attn", "achieved": round(achieved, 2),
             "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
