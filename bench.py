@@ -238,6 +238,24 @@ def run_gpu(args):
     per_launch_flops = attn_flops_total / len(ev)
     # all-frames-active comparison, same number of steps
     ms_all, _ = timed(core_all, K_steps, min(W_steps, 3))
+    # the step core's four launches, each timed on its own over one trajectory (latent width:
+    # the three small kernels are launch-bound, so their microseconds are reported, not GB/s)
+    parts = {"rf_schedule_compact": [], "rf_project": [], "rf_attn": [], "rf_step": []}
+    for k in range(S):
+        calls = (("rf_schedule_compact", lambda: core.compact(k)),
+                 ("rf_project", lambda: core.project(k)),
+                 ("rf_attn", lambda: core.attn(O, Q, K, V, w.softmax_scale)),
+                 ("rf_step", lambda: core.step(k, vel[k])))
+        for name, fn in calls:
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            parts[name].append((a, b))
+    barrier()
+    breakdown_us = {n: round(1000 * statistics.mean(a.elapsed_time(b) for a, b in v), 2)
+                    for n, v in parts.items()}
     # per schedule step: attention launch time against the all-active launch
     _, ev_all = timed(core_all, S, 3, per_launch=True)
     attn_all_ms = statistics.mean(a.elapsed_time(b) for _, a, b in ev_all)
@@ -305,6 +323,7 @@ def run_gpu(args):
         "ideal_speedup_vs_all_active": round(K_steps * flops_all /
                                              sum(flops_step[k % S] for k in range(K_steps)), 4),
         "per_step": per_step,
+        "step_core_breakdown_us": breakdown_us,
         "roofline": {
             "bound": "tensor", "kernel": "rf_attn", "achieved": round(achieved, 2),
             "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
