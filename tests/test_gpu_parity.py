@@ -780,3 +780,23 @@ def test_bandwidth_kernels_at_stress_shape_sampled(cuda_lib, name, s):
     stored = Kc[1 - sl, frames].reshape(w.F, E)[:, idx].cpu().double().numpy()
     np.testing.assert_array_equal(stored[m], kfresh[m])         # fresh rows shifted in
     np.testing.assert_array_equal(stored[sk], kprev[sk])        # skipped frames' cache kept
+
+
+def test_attn_block_masked_queue_with_several_head_groups(cuda_lib):
+    """A sequence long enough that only some heads' K/V fit in half of L2, so the longest-first
+    pre-pass orders the items in more than one group of heads (the last one smaller); a causal
+    block mask makes the costs differ.  Sampled rows of every head against the oracle, and a
+    second call on the same workspace (the group counters must be back at zero)."""
+    rf = cuda_lib
+    F, N, H, d = 2, 65536, 3, 64
+    Q, K, V = _qkv(F * N, H, d, seed=41)
+    nb = (F * N + 127) // 128
+    qb, kb = np.meshgrid(np.arange(nb), np.arange(nb), indexing="ij")
+    bm = np.broadcast_to((kb <= qb).astype(np.uint8), (H, nb, nb)).copy()
+    scale = 1.0 / math.sqrt(d)
+    rows = np.array([0, 127, 128, 5000, 65535, 65536, 70000, 100000, 131071])
+    for call in range(2):
+        O, L = _run_masked(rf, Q, K, V, F, N, [1, 1], scale, bm, split=True)
+        Oref, Lref = oracle.attention_block_masked(Q.cpu(), K.cpu(), V.cpu(), rows, scale, bm)
+        compare(O.cpu().float()[rows].numpy(), Oref, L.cpu()[:, rows].numpy(), Lref,
+                f"several head groups, call {call}")
