@@ -352,10 +352,11 @@ def run_gpu(args):
 
 
 def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist, world):
-    """End to end through the package's host pipeline: every step copies Q, K, V and the
-    velocity from pinned host memory and reads the attention output and the latent store
-    back, with the copies of neighbouring steps overlapped with compute (two copy streams,
-    double-buffered device inputs/outputs)."""
+    """End to end through the library's host-fed pipeline (rf_pipeline_step: one C-ABI call
+    per step, host pointers in and out).  Every step copies Q, K, V and the velocity from
+    pinned host memory and reads the attention output and the latent store back, with the
+    copies of neighbouring steps overlapped with compute (two copy streams, three device
+    buffer sets)."""
     import torch
     from paper_2606_06309_gb300.stepcore import HostPipeline
     S = w.S
@@ -379,9 +380,11 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
                                  float(sum(flops_step[k % S] for k in range(K_steps))), dist,
                                  Q.device)
     h2d, d2h = pipe.bytes_per_step(last=K_steps)
+    status = pipe.sync()
+    pipe.close()
     return {"value": round(flops / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "steps": K_steps,
             "ms_per_step": round(ms / K_steps, 5), "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h,
+            "d2h_bytes_per_step": d2h, "api": "rf_pipeline_step", "device_status": status,
             "overlap": "three buffer sets: H2D of steps k+1, k+2 and D2H of earlier steps "
                        "overlap the compute of step k",
             "copied": "in: active frames' Q rows, all of K and V, the velocity; out: active "

@@ -23,7 +23,9 @@
  * Conventions common to every call:
  *  - Pointers named d_* are device pointers, h_* host pointers.  The caller owns
  *    every buffer; no call allocates, frees or retains memory beyond its return
- *    (rf_attn keeps a small per-process cache of device properties only).
+ *    (rf_attn keeps a small per-process cache of device properties only), except
+ *    the host-fed pipeline object, which owns its device memory from
+ *    rf_pipeline_create to rf_pipeline_destroy.
  *  - `stream` is a cudaStream_t (NULL = the legacy default stream).  Work is
  *    enqueued and the call returns; nothing synchronises the host.
  *  - Errors that the host can see (null pointers, bad sizes, unsupported head
@@ -309,6 +311,54 @@ rf_status rf_frame_gram(const float* d_P, int F, int64_t E, int64_t ld, double* 
 rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double dtau,
                              double delta_up, double delta_down, uint8_t* h_is_key,
                              int32_t* h_num_keys);
+
+/*
+ * rf_pipeline -- the step core fed from pinned host memory: one asynchronous denoising step
+ * (Algorithm 2: rf_schedule_compact, rf_project, rf_attn, rf_step) per rf_pipeline_step,
+ * with the step's inputs copied from the host and its results copied back, the copies of
+ * neighbouring steps overlapped with the compute of the current one.  No paper passage: this
+ * is the host side of serving the step core.
+ *
+ * rf_pipeline_create allocates, on the current device, the plan, the two-slot latent store,
+ * the index lists, an rf_attn workspace and `depth` buffer sets (Q, K, V, O bf16
+ * [F*N][H][d]; velocity fp32 [F][E]; a latent-store snapshot fp32 [2][F][E]).
+ *   h_mask, h_alpha, h_beta, h_dt, h_cur_slot  the plan, [S][F] as rf_plan_build writes it
+ *   h_z2        fp32 [2][F][E] initial two-slot latent store
+ *   depth       buffer sets, 2..8 (3 lets a heavy step's input copies run during the two
+ *               steps before it)
+ *   compute, h2d, d2h  three streams the pipeline enqueues on (all work of a step is
+ *               ordered by events recorded on them; the caller may record its own events)
+ *   *out        the pipeline; RF_ERR_* and *out = NULL on failure (nothing leaks)
+ * d in {64, 128}; E % 4 == 0.
+ *
+ * rf_pipeline_step enqueues schedule step s (0 <= s < S) and returns:
+ *   h_Q, h_K, h_V  pinned host bf16 [F*N][H][d] (rows contiguous); only the rows of the
+ *               frames active at step s are read from h_Q
+ *   h_v         pinned host fp32 [F][E] velocity of the step
+ *   h_O         pinned host bf16 [F*N][H][d]: the active frames' rows are written
+ *   h_z2        pinned host fp32 [2][F][E]: the latent store after the step
+ *   softmax_scale  as for rf_attn
+ * Host buffers of a step must stay valid and untouched until rf_pipeline_sync; the buffers
+ * of `depth` consecutive steps may be in flight at once.
+ *
+ * rf_pipeline_sync waits for every enqueued step and writes the device status word (as for
+ * rf_attn) to *h_status (nullable).  rf_pipeline_bytes reports the steps enqueued and the
+ * host->device and device->host bytes they copy.  rf_pipeline_destroy waits and frees
+ * everything (NULL is ignored).
+ */
+typedef struct rf_pipeline rf_pipeline;
+rf_status rf_pipeline_create(int F, int N, int H, int d, int64_t E, int S,
+                             const uint8_t* h_mask, const float* h_alpha, const float* h_beta,
+                             const float* h_dt, const uint8_t* h_cur_slot, const float* h_z2,
+                             int depth, rf_stream_t compute, rf_stream_t h2d, rf_stream_t d2h,
+                             rf_pipeline** out);
+rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, const void* h_K,
+                           const void* h_V, const float* h_v, void* h_O, float* h_z2,
+                           float softmax_scale);
+rf_status rf_pipeline_sync(rf_pipeline* p, int32_t* h_status);
+rf_status rf_pipeline_bytes(const rf_pipeline* p, int64_t* h_steps, int64_t* h_h2d_bytes,
+                            int64_t* h_d2h_bytes);
+void rf_pipeline_destroy(rf_pipeline* p);
 
 /*
  * rf_selftest_bounded_wait -- check, on the GPU, the path every device-side wait

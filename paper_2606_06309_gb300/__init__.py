@@ -17,8 +17,9 @@ import numpy as np
 __all__ = ["load", "lib_path", "RFError", "rf_plan_build", "rf_schedule_compact",
            "rf_project", "rf_project_kv", "rf_attn", "rf_attn_block_masked",
            "rf_attn_workspace_bytes", "rf_attn_noalloc", "rf_step", "rf_frame_gram",
-           "rf_keyframe_select", "rf_selftest_bounded_wait", "rf_status_str", "rf_version",
-           "EXPORTS"]
+           "rf_keyframe_select", "rf_selftest_bounded_wait", "rf_pipeline_create",
+           "rf_pipeline_step", "rf_pipeline_sync", "rf_pipeline_bytes", "rf_pipeline_destroy",
+           "rf_status_str", "rf_version", "EXPORTS"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB: Optional[ctypes.CDLL] = None
@@ -28,7 +29,8 @@ EXPORTS = ("rf_status_str", "rf_version", "rf_last_error", "rf_plan_build",
            "rf_schedule_compact", "rf_project", "rf_project_kv", "rf_attn",
            "rf_attn_block_masked", "rf_attn_workspace_bytes",
            "rf_attn_noalloc", "rf_step", "rf_frame_gram", "rf_keyframe_select",
-           "rf_selftest_bounded_wait")
+           "rf_pipeline_create", "rf_pipeline_step", "rf_pipeline_sync", "rf_pipeline_bytes",
+           "rf_pipeline_destroy", "rf_selftest_bounded_wait")
 
 _vp, _i32, _i64, _f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
 _SIG = {
@@ -52,6 +54,12 @@ _SIG = {
     "rf_attn_noalloc": ([_vp, _vp, _vp, _vp, _vp, _i64, _i64, _i32, _i32, _i32, _i32, _vp, _vp,
                          _f32, _vp, _vp], _i32),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
+    "rf_pipeline_create": ([_i32, _i32, _i32, _i32, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
+                            _i32, _vp, _vp, _vp, ctypes.POINTER(_vp)], _i32),
+    "rf_pipeline_step": ([_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f32], _i32),
+    "rf_pipeline_sync": ([_vp, _vp], _i32),
+    "rf_pipeline_bytes": ([_vp, _vp, _vp, _vp], _i32),
+    "rf_pipeline_destroy": ([_vp], None),
 }
 
 
@@ -214,3 +222,48 @@ def rf_step(z2, cur_slot, v, dt, active, counts, F: int, E: int, stream=None):
     _check("rf_step", load().rf_step(
         _ptr(z2), _ptr(cur_slot), _ptr(v), _ptr(dt), _ptr(active), _ptr(counts), F, E,
         _stream(stream)))
+
+
+def rf_pipeline_create(F: int, N: int, H: int, d: int, E: int, plan: dict, z2, depth: int,
+                       compute, h2d, d2h) -> int:
+    """Host-fed step pipeline over the host plan (rf_plan_build's arrays) and an initial fp32
+    [2, F, E] latent store (host array or tensor); returns an opaque handle."""
+    # every array is bound to a name, so that none is freed before the call reads it
+    mask = np.ascontiguousarray(plan["mask"], dtype=np.uint8)
+    alpha = np.ascontiguousarray(plan["alpha"], dtype=np.float32)
+    beta = np.ascontiguousarray(plan["beta"], dtype=np.float32)
+    dt = np.ascontiguousarray(plan["dt"], dtype=np.float32)
+    slot = np.ascontiguousarray(plan["cur_slot"], dtype=np.uint8)
+    z = np.ascontiguousarray(np.asarray(z2.cpu() if hasattr(z2, "cpu") else z2), dtype=np.float32)
+    S = mask.shape[0]
+    out = _vp()
+    _check("rf_pipeline_create", load().rf_pipeline_create(
+        F, N, H, d, E, S, _ptr(mask), _ptr(alpha), _ptr(beta), _ptr(dt), _ptr(slot), _ptr(z),
+        depth, _stream(compute), _stream(h2d), _stream(d2h), ctypes.byref(out)))
+    return out.value
+
+
+def rf_pipeline_step(handle: int, s: int, hQ, hK, hV, hv, hO, hz2, softmax_scale: float):
+    _check("rf_pipeline_step", load().rf_pipeline_step(
+        handle, s, _ptr(hQ), _ptr(hK), _ptr(hV), _ptr(hv), _ptr(hO), _ptr(hz2),
+        float(softmax_scale)))
+
+
+def rf_pipeline_sync(handle: int) -> int:
+    """Wait for every enqueued step; returns the device status word."""
+    st = np.zeros(1, np.int32)
+    _check("rf_pipeline_sync", load().rf_pipeline_sync(handle, _ptr(st)))
+    return int(st[0])
+
+
+def rf_pipeline_bytes(handle: int):
+    """(steps, host->device bytes, device->host bytes) enqueued so far."""
+    v = np.zeros(3, np.int64)
+    _check("rf_pipeline_bytes", load().rf_pipeline_bytes(
+        handle, v.ctypes.data, v.ctypes.data + 8, v.ctypes.data + 16))
+    return int(v[0]), int(v[1]), int(v[2])
+
+
+def rf_pipeline_destroy(handle: int):
+    if handle:
+        load().rf_pipeline_destroy(handle)

@@ -20,8 +20,9 @@ from typing import Optional
 
 import torch
 
-from . import (rf_attn, rf_attn_workspace_bytes, rf_plan_build, rf_project, rf_schedule_compact,
-               rf_step)
+from . import (rf_attn, rf_attn_workspace_bytes, rf_pipeline_bytes, rf_pipeline_create,
+               rf_pipeline_destroy, rf_pipeline_step, rf_pipeline_sync, rf_plan_build, rf_project,
+               rf_schedule_compact, rf_step)
 
 
 @dataclass
@@ -118,18 +119,19 @@ class StepCore:
 class HostPipeline:
     """Step-core steps fed from pinned host memory, with the copies hidden behind compute.
 
-    Each step copies host -> device what the step reads: the query rows of the frames active
-    at that step (the attention reads no other query row), all of K and V (every query attends
-    to every key), and the velocity.  It copies device -> host what the step writes: the
-    active frames' rows of the attention output (no other row is written) and a snapshot of
-    the two-slot latent store.  Rows of consecutive active frames move in one copy each.
-    `depth` device buffer sets and two copy streams (one per direction, so both copy engines
-    work) let the input copies of the next depth-1 steps and the read-back of earlier steps
-    run during the compute of step k.  Events order the three streams; nothing synchronises
-    the host.  Three sets, not two: steps differ in cost (all frames active, then only the
-    keyframes), and with two sets the inputs of a heavy step could only be copied during the
-    short light step before it (0.84 ms of copies against 0.5 ms of compute on 13 x 1560
-    tokens).
+    A thin wrapper of the library's native pipeline (``rf_pipeline_*``), which owns the plan,
+    the two-slot latent store and `depth` device buffer sets.  Each step copies host -> device
+    what it reads: the query rows of the frames active at that step (the attention reads no
+    other query row), all of K and V, and the velocity.  It copies device -> host what it
+    writes: the active frames' rows of the attention output and a snapshot of the latent
+    store.  Three streams (compute, host->device, device->host) are ordered by events, so the
+    input copies of the next depth-1 steps and the read-back of earlier steps run during the
+    compute of step k; nothing synchronises the host.  Three sets, not two: steps differ in
+    cost (all frames active, then only the keyframes), and with two sets the inputs of a heavy
+    step could only be copied during the short light step before it (0.84 ms of copies against
+    0.5 ms of compute on 13 x 1560 tokens).
+
+    The pipeline starts from `core`'s plan and current latent store; it does not change `core`.
     """
 
     def __init__(self, core: StepCore, S_tok: int, device="cuda", depth: int = 3):
@@ -140,79 +142,37 @@ class HostPipeline:
         self.compute = torch.cuda.current_stream(dev)
         self.h2d = torch.cuda.Stream(dev)
         self.d2h = torch.cuda.Stream(dev)
-        H, d, F, E = core.H, core.d, core.F, core.E
-        self.buf = []
-        for _ in range(depth):
-            self.buf.append({
-                "Q": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
-                "K": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
-                "V": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
-                "v": torch.empty(F, E, dtype=torch.float32, device=dev),
-                "O": torch.empty(S_tok, H, d, dtype=torch.bfloat16, device=dev),
-                "z": torch.empty(2, F, E, dtype=torch.float32, device=dev),
-            })
-        ev = lambda: [torch.cuda.Event() for _ in range(depth)]
-        self.loaded = ev()     # inputs of buffer b are on the device
-        self.consumed = ev()   # compute finished with buffer b (inputs read, outputs ready)
-        self.drained = ev()    # outputs of buffer b are back on the host
-        self.k = 0
-        self.moved = []                # (host->device, device->host) bytes of each step
-
-    def active_runs(self, s: int):
-        """[f0, f1) ranges of consecutive frames active at schedule step s."""
-        m = self.core.plan.host["mask"][s]
-        runs, f, F = [], 0, len(m)
-        while f < F:
-            if m[f]:
-                g = f
-                while g < F and m[g]:
-                    g += 1
-                runs.append((f, g))
-                f = g
-            else:
-                f += 1
-        return runs
+        torch.cuda.synchronize(dev)  # the core's latent store is read below
+        self.handle = rf_pipeline_create(core.F, self.N, core.H, core.d, core.E, core.plan.host,
+                                         core.z2, depth, self.compute, self.h2d, self.d2h)
+        self._marks = []  # (steps, h2d bytes, d2h bytes) after each step
 
     def step(self, s: int, hQ, hK, hV, hv, hO, hz, scale: float):
         """Enqueue schedule step s: inputs from pinned host tensors hQ, hK, hV (bf16
-        [S_tok, H, d]) and hv (fp32 [F, E]); results into pinned hO (bf16; the active frames'
-        rows) and hz (fp32 [2, F, E]).  Returns immediately."""
-        b = self.k % self.depth
-        B = self.buf[b]
-        N = self.N
-        rows = [(f0 * N, f1 * N) for f0, f1 in self.active_runs(s)]
-        first_use = self.k < self.depth
-        with torch.cuda.stream(self.h2d):
-            if not first_use:
-                self.h2d.wait_event(self.consumed[b])   # step k-depth has read these inputs
-            for r0, r1 in rows:
-                B["Q"][r0:r1].copy_(hQ[r0:r1], non_blocking=True)
-            B["K"].copy_(hK, non_blocking=True)
-            B["V"].copy_(hV, non_blocking=True)
-            B["v"].copy_(hv, non_blocking=True)
-            self.loaded[b].record(self.h2d)
-        self.compute.wait_event(self.loaded[b])
-        if not first_use:
-            self.compute.wait_event(self.drained[b])    # step k-depth's outputs are on the host
-        self.core.run(s, B["v"], B["O"], B["Q"], B["K"], B["V"], scale, stream=self.compute)
-        B["z"].copy_(self.core.z2, non_blocking=True)
-        self.consumed[b].record(self.compute)
-        with torch.cuda.stream(self.d2h):
-            self.d2h.wait_event(self.consumed[b])
-            for r0, r1 in rows:
-                hO[r0:r1].copy_(B["O"][r0:r1], non_blocking=True)
-            hz.copy_(B["z"], non_blocking=True)
-            self.drained[b].record(self.d2h)
-        self.k += 1
-        nbytes = lambda t: t.numel() * t.element_size()
-        row_q = nbytes(B["Q"][0])
-        act = sum(r1 - r0 for r0, r1 in rows)
-        self.moved.append((act * row_q + nbytes(B["K"]) + nbytes(B["V"]) + nbytes(B["v"]),
-                           act * row_q + nbytes(B["z"])))
+        [S_tok, H, d], contiguous rows) and hv (fp32 [F, E]); results into pinned hO (bf16; the
+        active frames' rows) and hz (fp32 [2, F, E]).  Returns immediately."""
+        rf_pipeline_step(self.handle, s, hQ, hK, hV, hv, hO, hz, scale)
+        self._marks.append(rf_pipeline_bytes(self.handle))
+
+    def sync(self) -> int:
+        """Wait for every enqueued step; returns the device status word."""
+        return rf_pipeline_sync(self.handle)
 
     def bytes_per_step(self, last: Optional[int] = None):
         """Average (host->device, device->host) bytes of the last `last` steps (all steps if
         None)."""
-        moved = self.moved if last is None else self.moved[-last:]
-        n = max(1, len(moved))
-        return (int(round(sum(m[0] for m in moved) / n)), int(round(sum(m[1] for m in moved) / n)))
+        if not self._marks:
+            return 0, 0
+        n = len(self._marks) if last is None else min(last, len(self._marks))
+        end = self._marks[-1]
+        start = self._marks[-n - 1] if n < len(self._marks) else (0, 0, 0)
+        steps = end[0] - start[0]
+        return (int(round((end[1] - start[1]) / steps)), int(round((end[2] - start[2]) / steps)))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            rf_pipeline_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        self.close()

@@ -113,6 +113,34 @@ def test_device_calls_reject_bad_args_on_host(rf):
     assert lib.rf_attn_block_masked(*margs) == 2                      # 4097 key blocks
 
 
+def test_pipeline_rejects_bad_args_on_host(rf):
+    """The host-fed pipeline's argument checks run before any allocation or CUDA call."""
+    lib = rf.load()
+    P = 256
+    out = ctypes.c_void_p(12345)
+    pa = [4, 8, 2, 128, 64, 3, P, P, P, P, P, P, 3, None, None, None, ctypes.byref(out)]
+    bad = list(pa)
+    bad[16] = None
+    assert lib.rf_pipeline_create(*bad) == 1                          # no handle to write
+    bad = list(pa)
+    bad[6] = None
+    assert lib.rf_pipeline_create(*bad) == 1 and out.value is None    # null plan; handle cleared
+    bad = list(pa)
+    bad[3] = 96
+    assert lib.rf_pipeline_create(*bad) == 2                          # d = 96 unsupported
+    bad = list(pa)
+    bad[4] = 66
+    assert lib.rf_pipeline_create(*bad) == 3                          # E % 4 != 0
+    for depth in (1, 9):
+        bad = list(pa)
+        bad[12] = depth
+        assert lib.rf_pipeline_create(*bad) == 1                      # depth outside 2..8
+    assert lib.rf_pipeline_step(None, 0, P, P, P, P, P, P, 0.1) == 1
+    assert lib.rf_pipeline_sync(None, None) == 1
+    assert lib.rf_pipeline_bytes(None, None, None, None) == 1
+    lib.rf_pipeline_destroy(None)                                     # a no-op
+
+
 def _scene_proxies(F=21, E=960, starts=(0, 4, 9, 13, 17), noise=0.3, seed=0):
     rng = np.random.default_rng(seed)
     base = rng.standard_normal((len(starts), E))

@@ -387,14 +387,14 @@ def test_host_pipeline_matches_device_path(cuda_lib, name):
     hz = [torch.zeros(core.z2.shape).pin_memory() for _ in range(nsteps)]
     for s in range(nsteps):
         pipe.step(s, hQ, hK, hV, hv[s], hO[s], hz[s], w.softmax_scale)
-    torch.cuda.synchronize()
+    assert pipe.sync() == 0
     for s in range(nsteps):
         act = np.array(_active_rows(oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)["mask"][s], w.N))
         assert torch.equal(hO[s][act], outs[s][0][act]), s
         assert torch.equal(hz[s], outs[s][1]), s
         skipped = np.setdiff1d(np.arange(w.S_tok), act)
         assert (hO[s][skipped] == 0).all(), s      # rows no step writes are not copied back
-    assert core.status.item() == 0
+    pipe.close()
 
 
 # ---------------------------------------------------------------------------
