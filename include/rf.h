@@ -339,7 +339,9 @@ rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double
  *   h_z2        pinned host fp32 [2][F][E]: the latent store after the step
  *   softmax_scale  as for rf_attn
  * Host buffers of a step must stay valid and untouched until rf_pipeline_sync; the buffers
- * of `depth` consecutive steps may be in flight at once.
+ * of `depth` consecutive steps may be in flight at once.  A step that returns an error may
+ * have enqueued part of its work, and the order between later steps is then not kept: after
+ * an error, call rf_pipeline_sync (to drain) and rf_pipeline_destroy.
  *
  * rf_pipeline_sync waits for every enqueued step and writes the device status word (as for
  * rf_attn) to *h_status (nullable).  rf_pipeline_bytes reports the steps enqueued and the

@@ -354,10 +354,11 @@ def test_attn_split_and_unsplit_agree_with_oracle(cuda_lib, F, N, H, d, mask):
     assert (O1.float() - O2.float()).abs().max().item() < 1e-2
 
 
-@pytest.mark.parametrize("name", ["tiny", "small"])
-def test_host_pipeline_matches_device_path(cuda_lib, name):
-    """HostPipeline (inputs from pinned host memory, copies overlapped with compute) gives
-    exactly the outputs of the same steps run on device-resident inputs."""
+@pytest.mark.parametrize("name,depth", [("tiny", 2), ("tiny", 5), ("small", 3)])
+def test_host_pipeline_matches_device_path(cuda_lib, name, depth):
+    """The native host-fed pipeline (inputs from pinned host memory, copies overlapped with
+    compute, `depth` device buffer sets) gives exactly the outputs of the same steps run on
+    device-resident inputs, and counts the bytes it copies."""
     from paper_2606_06309_gb300.stepcore import HostPipeline, StepCore, upload_plan
     w = wl.get(name)
     E = w.N * w.C
@@ -380,7 +381,7 @@ def test_host_pipeline_matches_device_path(cuda_lib, name):
         outs.append((O.cpu().clone(), ref.z2.cpu().clone()))
 
     core = fresh()
-    pipe = HostPipeline(core, w.S_tok, DEV)
+    pipe = HostPipeline(core, w.S_tok, DEV, depth=depth)
     hQ, hK, hV = (x.cpu().pin_memory() for x in (Q, K, V))
     hv = [v.pin_memory() for v in vel]
     hO = [torch.zeros(Q.shape, dtype=Q.dtype).pin_memory() for _ in range(nsteps)]
@@ -394,7 +395,15 @@ def test_host_pipeline_matches_device_path(cuda_lib, name):
         assert torch.equal(hz[s], outs[s][1]), s
         skipped = np.setdiff1d(np.arange(w.S_tok), act)
         assert (hO[s][skipped] == 0).all(), s      # rows no step writes are not copied back
+    # bytes: active Q rows, K, V and v in; active O rows and both latent slots out
+    row = w.H * w.d * 2
+    n_act = sum(len(_active_rows(oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)["mask"][s],
+                                 w.N)) for s in range(nsteps))
+    h2d, d2h = pipe.bytes_per_step()
+    assert h2d == round((n_act * row + nsteps * (2 * w.S_tok * row + w.F * E * 4)) / nsteps)
+    assert d2h == round((n_act * row + nsteps * 2 * w.F * E * 4) / nsteps)
     pipe.close()
+    pipe.close()                                    # closing twice is harmless
 
 
 # ---------------------------------------------------------------------------
