@@ -259,6 +259,27 @@ def test_attn_planted_keys(cuda_lib):
     assert err < 2e-2, err
 
 
+@pytest.mark.parametrize("direction,mask,split", [
+    ("up", [1, 1, 1], True), ("up", [1, 0, 1], False), ("down", [1, 1, 1], False),
+    ("down", [0, 1, 1], True)])
+def test_attn_running_max_moves_across_tiles(cuda_lib, direction, mask, split):
+    """Keys scaled by a ramp along the sequence (x1 to x7), queries x2: with the ramp going up,
+    every row's running max keeps growing from one KV tile to the next, so the lazy rescale of
+    the accumulator fires many times per row and unnormalised p reaches 2^8 between rescales;
+    going down, the max is set by the first tiles and later tiles contribute tiny p."""
+    rf = cuda_lib
+    F, N, H, d = 3, 700, 2, 128
+    Q, K, V = _qkv(F * N, H, d, seed=71 if direction == "up" else 72)
+    ramp = torch.linspace(1.0, 7.0, F * N, device=DEV)
+    if direction == "down":
+        ramp = ramp.flip(0)
+    K = (K.float() * ramp[:, None, None]).to(torch.bfloat16)
+    Q = (2.0 * Q.float()).to(torch.bfloat16)
+    scale = 1.0 / math.sqrt(d)
+    O, L = _run_attn(rf, Q, K, V, F, N, mask, scale, split=split)
+    _check_attn(Q, K, V, O, L, mask, N, scale, label=f"ramp {direction} {mask} split={split}")
+
+
 @pytest.mark.parametrize("name,steps", [("small", (0, 1)), ("mid", (0, 18)), ("large", (0, 1)),
                                         ("long", (0, 12))])
 def test_attn_full_size_sampled_rows(cuda_lib, name, steps):
