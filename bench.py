@@ -615,66 +615,93 @@ def _cpu_model():
     return platform.machine() + (" (" + ", ".join(parts) + ")" if parts else "")
 
 
+class _OracleSample:
+    """One step of the fp64 oracle on a bounded sample, inputs prepared once: the schedule,
+    projection and Euler update for every frame at latent width, and attention for a given
+    number of sampled active query rows (all heads, all keys)."""
+
+    def __init__(self, w, s=0):
+        import numpy as np
+        import oracle
+        import workloads as wl
+        self.w, self.s = w, s
+        self.Q, self.K, self.V = wl.qkv(w)  # host copy of the same seeded inputs
+        self.plan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
+        mask = self.plan["mask"][s]
+        self.rows_all = np.array([f * w.N + p for f in range(w.F) if mask[f]
+                                  for p in range(w.N)])
+        self.z = wl.latents(w).double().numpy()
+        self.v = wl.velocity(w, s).double().numpy()
+        self.rng = np.random.default_rng(0)
+
+    def run(self, n_rows):
+        """(algorithmic attention FLOPs, seconds) of one sample step with n_rows query rows."""
+        import oracle
+        w, s = self.w, self.s
+        n = int(min(max(1, n_rows), len(self.rows_all)))
+        rows = self.rng.choice(self.rows_all, size=n, replace=False)
+        t0 = time.perf_counter()
+        oracle.compact(self.plan["mask"][s], w.N)
+        oracle.project(self.z, self.z, self.plan["alpha"][s])
+        oracle.euler(self.z, self.v, self.plan["dt"][s])
+        oracle.attention(self.Q, self.K, self.V, rows, w.softmax_scale)
+        return oracle.flops_attn(n, w.S_tok, w.d, w.H), time.perf_counter() - t0
+
+    def describe(self, flops):
+        w = self.w
+        return (f"step {self.s} of {w.name}: full schedule/projection/Euler at latent width plus "
+                f"attention of sampled active rows x {w.H} heads x {w.S_tok} keys (fp64 numpy, "
+                f"{flops / 1e12:.3f} TFLOP)")
+
+
 def cpu_baseline(w, budget_s=15.0):
-    """The fp64 oracle as it stands, on a bounded sample of one step: schedule,
-    projection and Euler update for every frame at latent width, and attention for a
-    growing number of sampled active query rows (all heads, all keys) until the budget
-    is spent.  Throughput is the sample's algorithmic attention FLOPs per second."""
-    import numpy as np
-    import torch
-    import oracle
-    import workloads as wl
-    Q, K, V = wl.qkv(w)  # host copy of the same seeded inputs
-    plan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
-    s = 0
-    mask = plan["mask"][s]
-    rows_all = np.array([f * w.N + p for f in range(w.F) if mask[f] for p in range(w.N)])
-    rng = np.random.default_rng(0)
-    z = wl.latents(w).double().numpy()
-    v = wl.velocity(w, s).double().numpy()
-    t0 = time.perf_counter()
-    oracle.compact(mask, w.N)
-    oracle.project(z, z, plan["alpha"][s])
-    oracle.euler(z, v, plan["dt"][s])
-    n, flops, elapsed = 64, 0, time.perf_counter() - t0
+    """The fp64 oracle as it stands, timed on the host cores: sample steps with a doubling
+    number of attention rows until the budget is spent.  Throughput is the samples'
+    algorithmic attention FLOPs per second."""
+    smp = _OracleSample(w)
+    n, flops, elapsed = 64, 0, 0.0
     while True:
-        rows = rng.choice(rows_all, size=min(n, len(rows_all)), replace=False)
-        t1 = time.perf_counter()
-        oracle.attention(Q, K, V, rows, w.softmax_scale)
-        elapsed += time.perf_counter() - t1
-        flops += oracle.flops_attn(len(rows), w.S_tok, w.d, w.H)
-        if elapsed >= budget_s or n >= len(rows_all):
+        f, t = smp.run(n)
+        flops += f
+        elapsed += t
+        if elapsed >= budget_s or n >= len(smp.rows_all):
             break
         n *= 2
     return {"value": round(flops / elapsed / 1e12, 6), "unit": UNIT, "cores": os.cpu_count(),
             "cpu": _cpu_model(), "kind": "oracle", "seconds": round(elapsed, 2),
-            "sample": f"step {s} of {w.name}: full schedule/projection/Euler at latent width "
-                      f"plus attention of sampled active rows x {w.H} heads x {w.S_tok} keys "
-                      f"(fp64 numpy, {flops / 1e12:.3f} TFLOP)"}
+            "sample": smp.describe(flops)}
 
 
 def run_reference(args):
+    """The reference arm: the oracle as it stands on the host cores.  Every step (warm-up
+    included) is one sample step of the same workload; the number of sampled attention rows is
+    set once, from a calibration sample, so that the whole run takes about two minutes
+    whatever --steps and --warmup are."""
     rank, world, _ = _env_rank()
     if rank != 0:
         return
     import workloads as wl
     w = wl.get(args.config)
-    vals = []
-    budget = max(2.0, min(20.0, 120.0 / max(1, args.steps + args.warmup)))
+    smp = _OracleSample(w)
+    f0, t0 = smp.run(64)                               # calibration (not counted)
+    per_step = min(20.0, 120.0 / max(1, args.steps + args.warmup))
+    n_rows = max(1, min(len(smp.rows_all), int(64 * per_step / max(t0, 1e-6))))
+    flops, secs = 0, 0.0
     for k in range(args.warmup + args.steps):
-        cb = cpu_baseline(w, budget_s=budget)
+        f, t = smp.run(n_rows)
         if k >= args.warmup:
-            vals.append(cb)
-    value = statistics.mean(c["value"] for c in vals)
-    secs = sum(c["seconds"] for c in vals)
+            flops += f
+            secs += t
+    value = round(flops / secs / 1e12, 6)
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup,
-           "ms_per_step": round(1000 * secs / len(vals), 3), "higher_is_better": True,
+           "ms_per_step": round(1000 * secs / max(1, args.steps), 3), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads "
                                   f"x {w.d}, latent {w.C} ch, {w.S} flow-matching steps"},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
-                            "cpu": vals[0]["cpu"], "kind": "oracle", "sample": vals[0]["sample"]},
+                            "cpu": _cpu_model(), "kind": "oracle",
+                            "sample": f"{n_rows} attention rows per step; " + smp.describe(flops)},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
