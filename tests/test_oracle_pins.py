@@ -107,6 +107,29 @@ def test_flop_example_step_counts():
     assert (asyn[~asyn.all(axis=1)].sum(axis=1) == M).all()
 
 
+def test_attention_flop_count_matches_printed_example():
+    """Appendix B.1 prints the attention FLOPs of one dense Wan 2.1 layer (S = 75,600 tokens,
+    D = 1,536 = 12 heads x 128) as 17.56 TFLOPs of 18.27, counting one FLOP per multiply-add.
+    The oracle's count (two per multiply-add, the one the benchmark divides by) is exactly twice
+    the printed attention term at full size."""
+    g = json.load(open(os.path.join(GOLDEN, "attention_flops_wan21.json")))
+    S, D = g["S"], g["D"]
+    attn_mac = oracle.flops_attn(S, S, g["head_dim"], g["heads"]) // 2   # S^2 D, twice
+    assert attn_mac == 2 * S * S * D
+    assert round(attn_mac / 1e12, 2) == g["printed_attention_tflops_per_layer"]
+    layer = 4 * S * D * D + attn_mac
+    assert round(layer / 1e12, 2) == g["printed_layer_tflops"]
+    assert round(100 * attn_mac / layer, 1) == g["printed_attention_share_pct"]
+    # skip-step layer: the printed projection term is within 0.2% of the formula's 4 S D^2; the
+    # printed attention term is exactly 4 S^2 D, twice the formula's 2 S^2 D (inconsistent
+    # figures of the paper; the oracle follows the formula)
+    Ss = g["S_skip"]
+    proj, attn = g["printed_skip_layer_terms"]
+    assert abs(proj / (4 * Ss * D * D) - 1) < 2e-3
+    assert oracle.flops_attn(Ss, Ss, g["head_dim"], g["heads"]) // 2 == 2 * Ss * Ss * D
+    assert attn == 2 * (2 * Ss * Ss * D)
+
+
 @pytest.mark.parametrize("n", [2, 3, 4, 5])
 def test_skip_count_identity(n):
     """Appendix B.1: N_skip = floor(T_R (n-1)/n) with T_R = 40."""
