@@ -427,6 +427,52 @@ def test_host_pipeline_matches_device_path(cuda_lib, name, depth):
     pipe.close()                                    # closing twice is harmless
 
 
+@pytest.mark.parametrize("F,N,H,d,keys,depth", [
+    (5, 100, 3, 64, [0, 3], 2),      # N % 8 != 0: padded query tiles, partial frames
+    (1, 37, 1, 128, [0], 4),         # one frame, a 37-token sequence (KV tail only)
+    (9, 24, 2, 128, [0, 4, 8], 8),   # the deepest buffer ring, more steps in flight than sets
+])
+def test_host_pipeline_ragged_shapes(cuda_lib, F, N, H, d, keys, depth):
+    """The native pipeline on ragged shapes gives the device path's outputs bit for bit."""
+    from paper_2606_06309_gb300.stepcore import HostPipeline, StepCore, upload_plan
+    S, E = 10, N * 16
+    is_key = [1 if f in keys else 0 for f in range(F)]
+    g = torch.Generator(device=DEV).manual_seed(F * 100 + N)
+    Q, K, V = (torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
+               for _ in range(3))
+    vel = [torch.randn(F, E, generator=g, device=DEV) for _ in range(S)]
+    z0 = torch.randn(F, E, generator=g, device=DEV)
+    scale = 1 / math.sqrt(d)
+
+    def fresh():
+        c = StepCore(F, N, E, H, d, upload_plan(F, S, is_key, [2] * S, 0, DEV), DEV)
+        c.set_state(z0)
+        return c
+
+    ref = fresh()
+    O = torch.zeros_like(Q)
+    outs = []
+    for s in range(S):
+        ref.run(s, vel[s], O, Q, K, V, scale)
+        outs.append((O.cpu().clone(), ref.z2.cpu().clone()))
+    assert ref.status.item() == 0
+    core = fresh()
+    pipe = HostPipeline(core, F * N, DEV, depth=depth)
+    hQ, hK, hV = (x.cpu().pin_memory() for x in (Q, K, V))
+    hv = [v.cpu().pin_memory() for v in vel]
+    hO = [torch.zeros(Q.shape, dtype=Q.dtype).pin_memory() for _ in range(S)]
+    hz = [torch.zeros(core.z2.shape).pin_memory() for _ in range(S)]
+    for s in range(S):
+        pipe.step(s, hQ, hK, hV, hv[s], hO[s], hz[s], scale)
+    assert pipe.sync() == 0
+    mask = oracle.schedule(F, S, is_key, [2] * S, 0)["mask"]
+    for s in range(S):
+        act = np.array(_active_rows(mask[s], N))
+        assert torch.equal(hO[s][act], outs[s][0][act]), s
+        assert torch.equal(hz[s], outs[s][1]), s
+    pipe.close()
+
+
 # ---------------------------------------------------------------------------
 # rf_project_kv: rolling key/value cache (Appendix B.2)
 # ---------------------------------------------------------------------------
