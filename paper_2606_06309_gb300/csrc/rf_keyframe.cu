@@ -9,7 +9,7 @@
 // Kernel: split-K over the proxy length E.  Each CTA of 256 threads owns a grid-stride set of
 // 128-element slices of every frame, stages them in shared memory k-major, and accumulates
 // partial products in registers (4 x 4 per thread, fp32) for the upper triangle of a tile of
-// 16, 24, 36, 48 or 64 frames (the smallest that holds F); at the end it adds its tile to the fp64 result with atomics.
+// 16, 24, 40, 48 or 64 frames (the smallest that holds F); at the end it adds its tile to the fp64 result with atomics.
 #include <cuda_runtime.h>
 
 #include "rf_host.h"
@@ -30,7 +30,7 @@ template <int TILE>
 __global__ void __launch_bounds__(kGramThreads)
     gram_kernel(const float* __restrict__ P, int F, int64_t E, int64_t ld, double* __restrict__ G) {
   constexpr int TG = (TILE / 4) * (TILE / 4);  // threads per k-group
-  static_assert(TILE % 4 == 0 && TG <= kGramThreads, "tile");
+  static_assert(TILE % 8 == 0 && TG <= kGramThreads && kGramK % 16 == 0, "tile");
   constexpr int KG = kGramThreads / TG;          // k-groups per CTA (leftover threads only load)
   constexpr int kStageV = TILE * kGramK / 4;     // float4 per stage
   constexpr int NV = (kStageV + kGramThreads - 1) / kGramThreads;  // per thread
@@ -43,11 +43,17 @@ __global__ void __launch_bounds__(kGramThreads)
   const bool vec_ok = (ld % 4 == 0) && ((reinterpret_cast<uintptr_t>(P) & 15) == 0);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kGramK;
   float4 pre[NV];
+  // float4 v of a stage -> (frame lf, element lk): a warp's 32 consecutive v cover 8 frames x 16
+  // elements (64 contiguous bytes per frame), so the transposed stores below spread over 16
+  // banks (2-way) where 32 rows of one frame column would fall into 2 banks (16-way)
+  auto frame_of = [](int v) { return ((v >> 5) % (TILE / 8)) * 8 + ((v & 31) >> 2); };
+  auto elem_of = [](int v) { return ((v >> 5) / (TILE / 8)) * 16 + (v & 3) * 4; };
   auto load = [&](int64_t k0) {
 #pragma unroll
     for (int q = 0; q < NV; ++q) {
-      const int idx = (threadIdx.x + q * kGramThreads) * 4;
-      const int lf = idx / kGramK, lk = idx % kGramK;
+      const int v = threadIdx.x + q * kGramThreads;
+      const int idx = v * 4;
+      const int lf = frame_of(v), lk = elem_of(v);
       const float* prow = P + static_cast<int64_t>(lf) * ld + k0 + lk;
       if (idx >= kStageV * 4) {
         pre[q] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -67,9 +73,9 @@ __global__ void __launch_bounds__(kGramThreads)
     __syncthreads();  // the previous stage has been consumed
 #pragma unroll
     for (int q = 0; q < NV; ++q) {
-      const int idx = (threadIdx.x + q * kGramThreads) * 4;
-      if (idx >= kStageV * 4) break;
-      const int lf = idx / kGramK, lk = idx % kGramK;
+      const int v = threadIdx.x + q * kGramThreads;
+      if (v * 4 >= kStageV * 4) break;
+      const int lf = frame_of(v), lk = elem_of(v);
       tile[lk][lf] = pre[q].x;
       tile[lk + 1][lf] = pre[q].y;
       tile[lk + 2][lf] = pre[q].z;
@@ -143,8 +149,8 @@ extern "C" rf_status rf_frame_gram(const float* d_P, int F, int64_t E, int64_t l
     gram_kernel<16><<<b, kGramThreads, 0, s>>>(d_P, F, E, ld, d_G);
   else if (F <= 24)
     gram_kernel<24><<<b, kGramThreads, 0, s>>>(d_P, F, E, ld, d_G);
-  else if (F <= 36)
-    gram_kernel<36><<<b, kGramThreads, 0, s>>>(d_P, F, E, ld, d_G);
+  else if (F <= 40)
+    gram_kernel<40><<<b, kGramThreads, 0, s>>>(d_P, F, E, ld, d_G);
   else if (F <= 48)
     gram_kernel<48><<<b, kGramThreads, 0, s>>>(d_P, F, E, ld, d_G);
   else
