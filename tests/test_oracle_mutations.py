@@ -19,6 +19,8 @@ PIN_CALLS = [
     (pins.test_every_trajectory_reaches_zero, {"name": "mid"}),
     (pins.test_warmup_all_active, {}),
     (pins.test_matches_algorithm2_rule_constant_stride, {"n": 3, "T_w": 8, "T": 50}),
+    (pins.test_eq2_two_level_stride_paper_defaults, {}),
+    (pins.test_attention_flop_count_matches_printed_example, {}),
     (pins.test_flop_example_step_counts, {}),
     (pins.test_skip_count_identity, {"n": 3}),
     (pins.test_last_jump_clamped_to_sigma_zero, {}),

@@ -53,6 +53,26 @@ def test_tiny_worked_example_alpha_dt():
     assert p["cur_slot"][:, 1].tolist() == [0, 1, 1, 0]
 
 
+def test_eq2_two_level_stride_paper_defaults():
+    """Eq. 2 with the paper's defaults (T = 50, T_w = 8, T_mid = T/2, n_small = 2,
+    n_large = 3), worked by hand with the due-step reading: a non-keyframe is updated on
+    every warm-up step 0..7, then every 2 steps while s < T - T_mid = 25 (8, 10, ..., 24;
+    the jump from 24 lands on 26), then every 3 steps (26, 29, ..., 47, the last jump clamped
+    to sigma = 0).  Its step sizes are the gaps to the next update, in sigma units."""
+    T, T_w = 50, 8
+    stride = [2] * 25 + [3] * 25
+    p = oracle.schedule(F=2, S=T, is_key=[1, 0], stride=stride, T_w=T_w)
+    active = [s for s in range(T) if p["mask"][s, 1]]
+    assert active == list(range(8)) + list(range(8, 25, 2)) + list(range(26, 48, 3))
+    nxt = active[1:] + [T]
+    for s, n in zip(active, nxt):
+        assert p["dt"][s, 1] == pytest.approx(-(n - s) / T, abs=1e-7)
+    assert p["mask"][:, 0].all()                       # the keyframe on every step
+    # a skipped step between 26 and 29 projects with alpha = (sigma_26 - sigma_s)/(3/50)
+    assert p["alpha"][27, 1] == pytest.approx(1 / 3, abs=1e-7)
+    assert p["alpha"][28, 1] == pytest.approx(2 / 3, abs=1e-7)
+
+
 @pytest.mark.parametrize("name", list(wl.WORKLOADS))
 def test_every_trajectory_reaches_zero(name):
     """Each frame's Euler steps sum to sigma_S - sigma_0 = -1, every frame is
