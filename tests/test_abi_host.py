@@ -141,6 +141,23 @@ def test_pipeline_rejects_bad_args_on_host(rf):
     lib.rf_pipeline_destroy(None)                                     # a no-op
 
 
+def test_python_binding_raises_with_status(rf):
+    """The binding turns a non-zero status into RFError carrying it, with the status name and
+    the library's last-error text in the message (host-side checks; no GPU is touched)."""
+    plan = rf.rf_plan_build(3, 4, [1, 0, 1], [2] * 4, 0)
+    z2 = np.zeros((2, 3, 16), np.float32)
+    with pytest.raises(rf.RFError) as e:
+        rf.rf_pipeline_create(3, 8, 2, 96, 16, plan, z2, 3, 0, 0, 0)   # head dim 96
+    assert e.value.status == 2 and "rf_pipeline_create" in str(e.value)
+    with pytest.raises(rf.RFError) as e:
+        rf.rf_pipeline_create(3, 8, 2, 64, 18, plan, z2, 3, 0, 0, 0)   # E % 4 != 0
+    assert e.value.status == 3
+    with pytest.raises(rf.RFError) as e:
+        rf.rf_pipeline_create(3, 8, 2, 64, 16, plan, z2, 1, 0, 0, 0)   # depth 1
+    assert e.value.status == 1
+    assert rf.rf_status_str(2) and rf.rf_status_str(99)
+
+
 def _scene_proxies(F=21, E=960, starts=(0, 4, 9, 13, 17), noise=0.3, seed=0):
     rng = np.random.default_rng(seed)
     base = rng.standard_normal((len(starts), E))
