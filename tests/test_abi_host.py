@@ -158,6 +158,25 @@ def test_python_binding_raises_with_status(rf):
     assert rf.rf_status_str(2) and rf.rf_status_str(99)
 
 
+def test_header_is_a_c_abi(rf, tmp_path):
+    """include/rf.h compiles as C (gcc -std=c11, warnings as errors) and a C program linked
+    against librf.so builds a plan and reads statuses through it; no GPU is used."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    exe = tmp_path / "plan_smoke"
+    lib_dir = os.path.dirname(rf.lib_path())
+    cmd = [gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"),
+           os.path.join(ROOT, "tests", "c_abi", "plan_smoke.c"), "-L", lib_dir, "-lrf",
+           f"-Wl,-rpath,{lib_dir}", "-o", str(exe)]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0 and r.stdout.startswith("ok"), (r.returncode, r.stdout, r.stderr)
+
+
 def _scene_proxies(F=21, E=960, starts=(0, 4, 9, 13, 17), noise=0.3, seed=0):
     rng = np.random.default_rng(seed)
     base = rng.standard_normal((len(starts), E))
