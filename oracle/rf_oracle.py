@@ -25,8 +25,15 @@ Citations name the paper's sections, equations and algorithms:
                        keys/values projected with Eq. 3 from the two cached states,
                        active frames' fresh keys/values shifted into the cache.
 * keyframe_select() -- Algorithm 1 (dynamic sequential keyframe selection),
-                       Eq. 1.  Parity partly unpinned: the paper gives no values
-                       for tau, delta tau, delta_up, delta_down.
+                       Eq. 1.  The paper gives no values for tau, delta tau,
+                       delta_up or delta_down; they are parameters, and the
+                       function is pinned by hand-worked cases (identical frames,
+                       orthogonal frames, two angle cases that fix the order of
+                       the threshold test and the direction of its adjustment).
+* sampler()         -- a whole trajectory of Algorithm 2 with given velocities
+                       (schedule, Eq. 3 context and Euler updates in order).
+* flops_attn()      -- the attention FLOP count, two per multiply-add; Appendix
+                       B.1 prints the same terms at one per multiply-add.
 
 Readings where the paper is silent or inconsistent are stated at each function.
 """
