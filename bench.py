@@ -393,9 +393,25 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
     h2d, d2h = pipe.bytes_per_step(last=K_steps)
     status = pipe.sync()
     pipe.close()
+    # this machine's host->device copy rate (pinned, 256 MB, after the timed region): the step's
+    # input copies take h2d / rate, which bounds the e2e figure where it exceeds the compute
+    src = torch.empty(64 * 2 ** 20, dtype=torch.float32).pin_memory()
+    dst = torch.empty_like(src, device=Q.device)
+    dst.copy_(src, non_blocking=True)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(5):
+        dst.copy_(src, non_blocking=True)
+    b.record()
+    torch.cuda.synchronize()
+    h2d_gbs = 5 * src.numel() * 4 / (a.elapsed_time(b) * 1e-3) / 1e9
+    del src, dst
     return {"value": round(flops / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "steps": K_steps,
             "ms_per_step": round(ms / K_steps, 5), "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "api": "rf_pipeline_step", "device_status": status,
+            "h2d_gbs_measured": round(h2d_gbs, 1),
+            "h2d_ms_per_step_at_that_rate": round(h2d / (h2d_gbs * 1e9) * 1e3, 4),
             "overlap": "three buffer sets: H2D of steps k+1, k+2 and D2H of earlier steps "
                        "overlap the compute of step k",
             "copied": "in: active frames' Q rows, all of K and V, the velocity; out: active "
