@@ -6,8 +6,16 @@ tighter checks are added: relative Frobenius error <= 1e-2, |delta LSE| <= 1e-3,
 and (in the planted-key tests) O(1)-scale outputs.  The arithmetic that sets
 them: the kernel rounds O to bf16 (relative 2^-9 ~ 2e-3), rounds the
 probabilities to bf16 before the PV product (relative 2^-9 per term, averaging
-down over thousands of keys), accumulates in fp32 and evaluates exp2 with the
-hardware approximation (relative ~2^-22).
+down over thousands of keys, but not on rows dominated by a few keys),
+accumulates in fp32 and evaluates exp2 with the hardware approximation
+(relative ~2^-22).
+
+The max-abs bound is read relative to the output's magnitude where |O| > 1:
+|g - o| <= 2e-2 * max(1, |o|).  bf16 keeps 8 significant bits, so an output of
+4.25 is stored to within half an ulp of 0.0156 and one of 8 or more only to
+within 0.031: an absolute 2e-2 cannot hold there for any bf16 result.  Rows
+with |O| of several units occur where a few large keys dominate (the 21 x 3600
+workload's tokens with std 2).
 """
 import numpy as np
 
@@ -24,8 +32,11 @@ def compare(o_gpu, o_ref, lse_gpu=None, lse_ref=None, label=""):
     assert np.isfinite(g).all(), f"{label}: non-finite output"
     err = np.abs(g - r)
     rel = np.linalg.norm(g - r) / max(np.linalg.norm(r), 1e-30)
-    msg = f"{label}: max {err.max():.3e} mean {err.mean():.3e} relF {rel:.3e}"
-    assert err.max() <= MAX_ABS, msg
+    ratio = err / (MAX_ABS * np.maximum(1.0, np.abs(r)))
+    i = np.unravel_index(np.argmax(ratio), ratio.shape)
+    msg = (f"{label}: max {err.max():.3e}, worst against the bound {ratio[i]:.2f} "
+           f"(gpu {g[i]:.5f}, oracle {r[i]:.5f}) mean {err.mean():.3e} relF {rel:.3e}")
+    assert ratio.max() <= 1.0, msg
     assert err.mean() <= MEAN_ABS, msg
     assert rel <= REL_FRO, msg
     if lse_gpu is not None:

@@ -315,14 +315,13 @@ def test_attn_equal_scores_give_the_mean_of_v(cuda_lib):
 def test_attn_full_size_sampled_rows(cuda_lib, name, steps):
     """The benchmark's launch configuration at full size; sampled rows of every head against
     the oracle: the first and last row of every active frame, the rows around each 128-row
-    tile boundary of the first frame, and seeded random rows, 512 rows in all (128 on the
-    two largest workloads, where the fp64 oracle is slowest)."""
+    tile boundary of the first frame, and seeded random rows, 512 rows in all."""
     rf = cuda_lib
     w = wl.get(name)
     Q, K, V = wl.qkv(w, device=DEV)
     p = _plan(rf, w)
     heads = list(range(w.H))
-    n_rows = 128 if w.S_tok * w.H > 2_000_000 else 512
+    n_rows = 512
     rng = np.random.default_rng(w.seed)
     for s in steps:
         mask = p["mask"][s]
