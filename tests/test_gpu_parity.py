@@ -349,6 +349,23 @@ def test_attn_full_size_sampled_rows(cuda_lib, name, steps):
         assert (written == expect).all()
 
 
+@pytest.mark.parametrize("s", [0, 1])
+def test_attn_small_every_row_of_two_heads(cuda_lib, s):
+    """Every active row of the first and last head of the 13 x 1560-token workload, against
+    the fp64 oracle, in the benchmark's launch configuration (split-KV workspace)."""
+    rf = cuda_lib
+    w = wl.get("small")
+    Q, K, V = wl.qkv(w, device=DEV)
+    p = _plan(rf, w)
+    mask = p["mask"][s]
+    O, L = _run_attn(rf, Q, K, V, w.F, w.N, mask, w.softmax_scale)
+    rows = _active_rows(mask, w.N)
+    heads = [0, w.H - 1]
+    Oref, Lref = oracle.attention(Q.cpu(), K.cpu(), V.cpu(), rows, w.softmax_scale, heads)
+    compare(O.cpu().float()[rows][:, heads].numpy(), Oref, L.cpu()[heads][:, rows].numpy(),
+            Lref, f"small s={s} every row, heads {heads}")
+
+
 # ---------------------------------------------------------------------------
 # Whole trajectory: compaction + projection + attention + Euler step, S steps
 # ---------------------------------------------------------------------------
