@@ -723,6 +723,40 @@ def _check_masked(Q, K, V, O, L, mask, N, scale, bmask, label):
         assert (O.cpu()[torch.tensor(skipped[:4096])].float() == SENTINEL).all()
 
 
+@pytest.mark.parametrize("name,kind", [("mid", "band"), ("large", "band"), ("large", "causal")])
+def test_attn_block_masked_full_size_sampled(cuda_lib, name, kind):
+    """Block-masked attention at full size, through the longest-first work queue (workspace):
+    the benchmark's banded mask (|qb - kb| <= nb / 8) and a causal block mask (items from one
+    key tile to all of them), schedule steps 0 and 1.  Sampled rows: 512 of every head on
+    13/21 x 1560 tokens; on 21 x 3600 tokens x 40 heads, 128 rows of four heads spread over
+    the head range (the masked oracle gathers each row's allowed keys, 5-12 ms per row and
+    head there)."""
+    rf = cuda_lib
+    w = wl.get(name)
+    Q, K, V = wl.qkv(w, device=DEV)
+    p = _plan(rf, w)
+    nb = (w.S_tok + 127) // 128
+    qb, kb = np.meshgrid(np.arange(nb), np.arange(nb), indexing="ij")
+    allow = (np.abs(qb - kb) <= max(1, nb // 8)) if kind == "band" else (kb <= qb)
+    bmask = np.broadcast_to(allow.astype(np.uint8), (w.H, nb, nb)).copy()
+    big = w.S_tok * w.H > 2_000_000
+    n_rows = 128 if big else 512
+    heads = [0, w.H // 3, 2 * w.H // 3, w.H - 1] if big else list(range(w.H))
+    rng = np.random.default_rng(w.seed + 7)
+    for s in (0, 1):
+        mask = p["mask"][s]
+        O, L = _run_masked(rf, Q, K, V, w.F, w.N, mask, w.softmax_scale, bmask)
+        all_rows = np.array(_active_rows(mask, w.N))
+        rows = {int(r) for f in range(w.F) if mask[f] for r in (f * w.N, f * w.N + w.N - 1)}
+        rest = np.setdiff1d(all_rows, np.array(sorted(rows)))
+        rows.update(rng.choice(rest, size=n_rows - len(rows), replace=False).tolist())
+        rows = sorted(rows)
+        Oref, Lref = oracle.attention_block_masked(Q.cpu(), K.cpu(), V.cpu(), rows,
+                                                   w.softmax_scale, bmask, heads=heads)
+        compare(O.cpu().float()[rows][:, heads].numpy(), Oref, L.cpu()[heads][:, rows].numpy(),
+                Lref, f"{name} {kind} s={s}")
+
+
 @pytest.mark.parametrize("F,N,H,d,mask,density,split", [
     (4, 256, 2, 128, [1, 1, 1, 1], 0.5, True),
     (4, 256, 2, 128, [1, 0, 0, 1], 0.3, False),
