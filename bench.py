@@ -1,11 +1,12 @@
 """Benchmark of the RhymeFlow asynchronous step core on GB300.
 
-A "step" is one asynchronous denoising step of the trajectory, all four
-library calls (compaction, Eq. 3 projection, active-query attention, Euler
-update) over the workload's synthetic inputs resident in HBM.  Timed step k is
+A "step" is one asynchronous denoising step of the trajectory, all five
+library calls (compaction, Eq. 3 projection of the latents, Eq. 3 projection of
+the skipped frames' keys and values from the rolling cache, active-query
+attention, Euler update) over the workload's synthetic inputs resident in HBM.  Timed step k is
 schedule step s = k mod S, so K = S steps is one whole trajectory.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--config small]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config long]
     python bench.py --impl reference ...   # the CPU oracle on the host cores
 
 value        attention TFLOP/s of the whole step core (algorithmic FLOPs
@@ -36,12 +37,14 @@ METRIC = "rf_attn TFLOP/s (% BF16 peak); step-core ms vs all-frames-active on 1 
 UNIT = "TFLOP/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM traffic of one rf_attn launch measured with ncu (dram__bytes_read.sum +
-# dram__bytes_write.sum; the capture is summarised in profiles/attn_kernel_small_all_active.md).
-# It is reported only while the kernel source still has this hash.
-ATTN_TRAFFIC = {"code_sha256_rf_attn_cu": "1dbc04774a003efa85ab66865e238dc33cd685c42928fb7b7c8cc510260628ac",
-                "workload": "small", "bytes_per_launch": 187693568 + 46976768,
-                "launch": "schedule step 0 of the small workload (all 13 frames active)"}
+# DRAM traffic of rf_attn launches measured with ncu (dram__bytes_read.sum +
+# dram__bytes_write.sum), per workload.  A figure is reported only while the kernel source
+# still has the hash it was measured with.
+ATTN_TRAFFIC = {
+    "small": {"code_sha256_rf_attn_cu": "1dbc04774a003efa85ab66865e238dc33cd685c42928fb7b7c8cc510260628ac",
+              "bytes_per_launch": 187693568 + 46976768,
+              "launch": "schedule step 0 of the small workload (all 13 frames active)"},
+}
 
 
 def _env_rank():
@@ -175,6 +178,7 @@ def run_gpu(args):
     core = StepCore(w.F, w.N, E, w.H, w.d, plan, dev)
     core.set_state(wl.latents(w, device=dev))
     Q, K, V = wl.qkv(w, device=dev)
+    core.set_kv_cache(K, V)
     O = torch.empty_like(Q)
     vel = [wl.velocity(w, s, device=dev) for s in range(S)]
     stream = torch.cuda.current_stream(dev)
@@ -186,6 +190,7 @@ def run_gpu(args):
     plan_all = upload_plan(w.F, w.S, [1] * w.F, [1] * S, 0, dev)
     core_all = StepCore(w.F, w.N, E, w.H, w.d, plan_all, dev)
     core_all.set_state(wl.latents(w, device=dev))
+    core_all.set_kv_cache(K, V)
     flops_all = 4 * w.F * w.N * w.S_tok * w.d * w.H
 
     def barrier():
@@ -206,6 +211,7 @@ def run_gpu(args):
             s = k % S
             c.compact(s)
             c.project(s)
+            c.project_kv(s, K, V)
             if per_launch:
                 a = torch.cuda.Event(enable_timing=True)
                 b = torch.cuda.Event(enable_timing=True)
@@ -238,12 +244,14 @@ def run_gpu(args):
     per_launch_flops = attn_flops_total / len(ev)
     # all-frames-active comparison, same number of steps
     ms_all, _ = timed(core_all, K_steps, min(W_steps, 3))
-    # the step core's four launches, each timed on its own over one trajectory (latent width:
-    # the three small kernels are launch-bound, so their microseconds are reported, not GB/s)
-    parts = {"rf_schedule_compact": [], "rf_project": [], "rf_attn": [], "rf_step": []}
+    # the step core's five launches, each timed on its own over one trajectory (the latent-width
+    # kernels are launch-bound, so their microseconds are reported, not GB/s)
+    parts = {"rf_schedule_compact": [], "rf_project": [], "rf_project_kv": [], "rf_attn": [],
+             "rf_step": []}
     for k in range(S):
         calls = (("rf_schedule_compact", lambda: core.compact(k)),
                  ("rf_project", lambda: core.project(k)),
+                 ("rf_project_kv", lambda: core.project_kv(k, K, V)),
                  ("rf_attn", lambda: core.attn(O, Q, K, V, w.softmax_scale)),
                  ("rf_step", lambda: core.step(k, vel[k])))
         for name, fn in calls:
@@ -295,8 +303,9 @@ def run_gpu(args):
     peaks, peak_src = _peaks()
     traffic = None
     attn_src = os.path.join(ROOT, "paper_2606_06309_gb300", "csrc", "rf_attn.cu")
-    if ATTN_TRAFFIC["code_sha256_rf_attn_cu"] == _code_sha(attn_src) and args.config == ATTN_TRAFFIC["workload"]:
-        traffic = ATTN_TRAFFIC["bytes_per_launch"]
+    tr = ATTN_TRAFFIC.get(args.config)
+    if tr is not None and tr["code_sha256_rf_attn_cu"] == _code_sha(attn_src):
+        traffic = tr["bytes_per_launch"]
     bw = run_bandwidth(w, dev, peaks) if not args.no_bandwidth else None
     sweep = run_sweep(w, dev, Q, K, V, O, vel, max(3, min(K_steps, 10))) if w.sweep else None
     block = run_block_mask(w, dev, Q, K, V, O, plan, core) if not args.no_bandwidth else None
@@ -308,8 +317,7 @@ def run_gpu(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": {
-            "workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads x {w.d}, "
-                        f"latent {w.C} ch, {w.S} flow-matching steps",
+            "workload": _workload_name(w),
             "keyframes": list(w.keyframes), "stride": f"{w.stride[0]}..{w.stride[-1]}",
             "active_frames_per_step_avg": float(A_per_step.mean()),
             "l2": _l2_note(3 * Q.numel() * 2, dev),
@@ -330,7 +338,7 @@ def run_gpu(args):
             "frac": round(achieved / peaks["bf16_tflops"], 4),
             "frac_of_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4),
             "traffic": traffic,
-            "traffic_launch": ATTN_TRAFFIC["launch"] if traffic is not None else None,
+            "traffic_launch": tr["launch"] if traffic is not None else None,
             "flops_per_launch": per_launch_flops,
             "avg_launch_ms": round(attn_ms_total / len(ev), 5),
         },
@@ -338,7 +346,7 @@ def run_gpu(args):
         "active_fraction_sweep": sweep,
         "combined_block_mask": block,
         "e2e": e2e,
-        "gpu_launches": 4 * K_steps,
+        "gpu_launches": core.launches_per_step * K_steps,
         "clocks": clocks,
         "device_status": status,
     }
@@ -364,10 +372,10 @@ def _l2_note(qkv_bytes, dev):
 
 def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist, world):
     """End to end through the library's host-fed pipeline (rf_pipeline_step: one C-ABI call
-    per step, host pointers in and out).  Every step copies Q, K, V and the velocity from
-    pinned host memory and reads the attention output and the latent store back, with the
-    copies of neighbouring steps overlapped with compute (two copy streams, three device
-    buffer sets)."""
+    per step, host pointers in and out).  Every step copies the active frames' Q, K and V rows
+    and the velocity from pinned host memory and reads the attention output's active rows,
+    the latent context and the latent store back, with the copies of neighbouring steps
+    overlapped with compute (two copy streams, three device buffer sets)."""
     import torch
     from paper_2606_06309_gb300.stepcore import HostPipeline
     S = w.S
@@ -375,16 +383,17 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
     hv = [v.cpu().pin_memory() for v in vel]
     hO = torch.empty(Q.shape, dtype=Q.dtype).pin_memory()
     hz = torch.empty(core.z2.shape, dtype=core.z2.dtype).pin_memory()
-    pipe = HostPipeline(core, w.S_tok, Q.device)
+    hc = torch.empty(core.ctx.shape, dtype=core.ctx.dtype).pin_memory()
+    pipe = HostPipeline(core, w.S_tok, hK, hV, Q.device)
     K_steps = max(1, min(args.steps, args.e2e_steps))
     for k in range(3):
-        pipe.step(k % S, hQ, hK, hV, hv[k % S], hO, hz, w.softmax_scale)
+        pipe.step(k % S, hQ, hK, hV, hv[k % S], hO, hz, w.softmax_scale, hctx=hc)
     barrier()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(pipe.h2d)
     for k in range(K_steps):
-        pipe.step(k % S, hQ, hK, hV, hv[k % S], hO, hz, w.softmax_scale)
+        pipe.step(k % S, hQ, hK, hV, hv[k % S], hO, hz, w.softmax_scale, hctx=hc)
     t1.record(pipe.d2h)
     barrier()
     ms, flops, _ = combine_ranks(t0.elapsed_time(t1),
@@ -414,8 +423,10 @@ def run_e2e(args, w, core, plan, Q, K, V, vel, flops_step, stream, barrier, dist
             "h2d_ms_per_step_at_that_rate": round(h2d / (h2d_gbs * 1e9) * 1e3, 4),
             "overlap": "three buffer sets: H2D of steps k+1, k+2 and D2H of earlier steps "
                        "overlap the compute of step k",
-            "copied": "in: active frames' Q rows, all of K and V, the velocity; out: active "
-                      "frames' O rows, the latent store (bytes averaged over the timed steps)"}
+            "copied": "in: active frames' Q, K and V rows, the velocity (skipped frames' keys "
+                      "and values are projected from the device-resident cache); out: active "
+                      "frames' O rows, the latent context, the latent store (bytes averaged "
+                      "over the timed steps)"}
 
 
 def run_bandwidth(w, dev, peaks):
@@ -586,6 +597,7 @@ def run_sweep(w, dev, Q, K, V, O, vel, steps):
         t = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
         plan = Plan(t["mask"], t["alpha"], t["beta"], t["dt"], t["cur_slot"], host)
         core = StepCore(w.F, w.N, E, w.H, w.d, plan, dev)
+        core.set_kv_cache(K, V)
         for k in range(3):
             core.run(k % w.S, vel[k % w.S], O, Q, K, V, w.softmax_scale)
         torch.cuda.synchronize()
@@ -633,15 +645,16 @@ def _cpu_model():
 
 class _OracleSample:
     """One step of the fp64 oracle on a bounded sample, inputs prepared once: the schedule,
-    projection and Euler update for every frame at latent width, and attention for a given
-    number of sampled active query rows (all heads, all keys)."""
+    projection and Euler update for every frame at latent width, and attention for sampled
+    active query rows of sampled heads (all keys)."""
 
     def __init__(self, w, s=0):
         import numpy as np
         import oracle
         import workloads as wl
         self.w, self.s = w, s
-        self.Q, self.K, self.V = wl.qkv(w)  # host copy of the same seeded inputs
+        # the same seeded inputs, widened to fp64 once: the oracle takes fp64 arrays as they are
+        self.Q, self.K, self.V = (oracle.to_f64(x) for x in wl.qkv(w))
         self.plan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
         mask = self.plan["mask"][s]
         self.rows_all = np.array([f * w.N + p for f in range(w.F) if mask[f]
@@ -650,24 +663,28 @@ class _OracleSample:
         self.v = wl.velocity(w, s).double().numpy()
         self.rng = np.random.default_rng(0)
 
-    def run(self, n_rows):
-        """(algorithmic attention FLOPs, seconds) of one sample step with n_rows query rows."""
+    def run(self, n_rows, n_heads=None):
+        """(algorithmic attention FLOPs, seconds) of one sample step with n_rows query rows of
+        n_heads heads (all heads if None)."""
         import oracle
         w, s = self.w, self.s
         n = int(min(max(1, n_rows), len(self.rows_all)))
+        nh = w.H if n_heads is None else int(min(max(1, n_heads), w.H))
         rows = self.rng.choice(self.rows_all, size=n, replace=False)
+        heads = None if nh == w.H else sorted(self.rng.choice(w.H, size=nh, replace=False))
         t0 = time.perf_counter()
         oracle.compact(self.plan["mask"][s], w.N)
         oracle.project(self.z, self.z, self.plan["alpha"][s])
         oracle.euler(self.z, self.v, self.plan["dt"][s])
-        oracle.attention(self.Q, self.K, self.V, rows, w.softmax_scale)
-        return oracle.flops_attn(n, w.S_tok, w.d, w.H), time.perf_counter() - t0
+        oracle.attention(self.Q, self.K, self.V, rows, w.softmax_scale, heads)
+        return oracle.flops_attn(n, w.S_tok, w.d, nh), time.perf_counter() - t0
 
-    def describe(self, flops):
+    def describe(self, flops, n_heads=None):
         w = self.w
+        hs = f"{w.H} heads" if n_heads in (None, w.H) else f"{n_heads} sampled heads of {w.H}"
         return (f"step {self.s} of {w.name}: full schedule/projection/Euler at latent width plus "
-                f"attention of sampled active rows x {w.H} heads x {w.S_tok} keys (fp64 numpy, "
-                f"{flops / 1e12:.3f} TFLOP)")
+                f"attention of sampled active rows x {hs} x {w.S_tok} keys (fp64 numpy, inputs "
+                f"widened once; {flops / 1e12:.4f} TFLOP)")
 
 
 def cpu_baseline(w, budget_s=15.0):
@@ -690,21 +707,22 @@ def cpu_baseline(w, budget_s=15.0):
 
 def run_reference(args):
     """The reference arm: the oracle as it stands on the host cores.  Every step (warm-up
-    included) is one sample step of the same workload; the number of sampled attention rows is
-    set once, from a calibration sample, so that the whole run takes about two minutes
-    whatever --steps and --warmup are."""
+    included) is one sample step of the same workload; the numbers of sampled heads and
+    attention rows are set once, from a calibration sample (64 rows of one head), so that the
+    whole run takes about two minutes whatever --steps and --warmup are."""
     rank, world, _ = _env_rank()
     if rank != 0:
         return
     import workloads as wl
     w = wl.get(args.config)
     smp = _OracleSample(w)
-    f0, t0 = smp.run(64)                               # calibration (not counted)
+    f0, t1 = smp.run(64, 1)                            # calibration (not counted)
     per_step = min(20.0, 120.0 / max(1, args.steps + args.warmup))
-    n_rows = max(1, min(len(smp.rows_all), int(64 * per_step / max(t0, 1e-6))))
+    n_heads = max(1, min(w.H, int(per_step / max(t1, 1e-6))))
+    n_rows = max(1, min(len(smp.rows_all), int(64 * per_step / max(n_heads * t1, 1e-6))))
     flops, secs = 0, 0.0
     for k in range(args.warmup + args.steps):
-        f, t = smp.run(n_rows)
+        f, t = smp.run(n_rows, n_heads)
         if k >= args.warmup:
             flops += f
             secs += t
@@ -713,34 +731,92 @@ def run_reference(args):
            "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": round(1000 * secs / max(1, args.steps), 3), "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads "
-                                  f"x {w.d}, latent {w.C} ch, {w.S} flow-matching steps"},
+           "config": {"workload": _workload_name(w)},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
                             "cpu": _cpu_model(), "kind": "oracle",
-                            "sample": f"{n_rows} attention rows per step; " + smp.describe(flops)},
+                            "sample": f"{n_rows} attention rows per step; "
+                                      + smp.describe(flops, n_heads)},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
 
 
+def _workload_name(w):
+    return (f"{w.name}: {w.F} latent frames x {w.N} tokens, {w.H} heads x {w.d}, latent {w.C} "
+            f"ch, {w.S} flow-matching steps")
+
+
+def run_attn_shape(args):
+    """rf_attn alone at a given shape F,N,H,d with every frame active, random bf16 inputs
+    resident on the device and the split-KV workspace: the median launch time and TFLOP/s
+    (4 * F*N * F*N * d * H per launch).  A small fixed command for shapes outside the
+    workloads and for profiling one kernel."""
+    import torch
+    import paper_2606_06309_gb300 as rf
+    F, N, H, d = (int(x) for x in args.attn_shape.split(","))
+    rf.load()
+    dev = torch.device("cuda", 0)
+    S_tok = F * N
+    g = torch.Generator(device=dev).manual_seed(0)
+    Q, K, V = (torch.randn(S_tok, H, d, generator=g, device=dev).to(torch.bfloat16)
+               for _ in range(3))
+    O = torch.empty_like(Q)
+    ws = torch.zeros((rf.rf_attn_workspace_bytes(d) + 3) // 4, dtype=torch.int32, device=dev)
+    act = torch.zeros(F, dtype=torch.int32, device=dev)
+    skp = torch.zeros_like(act)
+    cnt = torch.zeros(2, dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    rf.rf_schedule_compact(torch.ones(F, dtype=torch.uint8, device=dev), F, N, act, skp, None,
+                           cnt)
+    scale = 1.0 / math.sqrt(d)
+    times = []
+    for _ in range(args.launches):
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        rf.rf_attn(O, None, Q, K, V, Q.stride(0), O.stride(0), F, N, H, d, act, cnt, scale, ws,
+                   status)
+        t1.record()
+        torch.cuda.synchronize()
+        times.append(t0.elapsed_time(t1))
+    ms = statistics.median(times[min(2, len(times) - 1):])
+    flops = 4 * S_tok * S_tok * d * H
+    st = int(status.item())
+    print(json.dumps({"attn_shape": {"F": F, "N": N, "H": H, "d": d}, "launches": args.launches,
+                      "median_ms": round(ms, 5), "tflops": round(flops / ms / 1e9, 1),
+                      "device_status": st}), flush=True)
+    if st != 0:
+        raise SystemExit(1)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=400)
-    ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--config", default="small")
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default: two whole trajectories of the workload)")
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="long",
+                    help="workload: tiny, small, mid, large or long (the largest, the default)")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-bandwidth", action="store_true")
     ap.add_argument("--bandwidth-only", action="store_true",
                     help="only the bandwidth-kernel leg (for profiling); prints its JSON")
+    ap.add_argument("--attn-shape", default=None, metavar="F,N,H,D",
+                    help="only rf_attn at this shape, every frame active (for profiling)")
+    ap.add_argument("--launches", type=int, default=10, help="launches for --attn-shape")
     args = ap.parse_args()
+    if args.steps is None:
+        import workloads as wl
+        args.steps = 2 * wl.get(args.config).S
     if args.warmup < 3 and args.impl != "reference":
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.attn_shape:
+        run_attn_shape(args)
     elif args.bandwidth_only:
         import torch
         import workloads as wl

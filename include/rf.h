@@ -9,11 +9,13 @@
  * linear projection of their latent trajectory (Eq. 3).  Afterwards only the
  * active frames take their Euler step.
  *
- * One step of that core is four calls, all asynchronous on a caller-provided
+ * One step of that core is five calls, all asynchronous on a caller-provided
  * CUDA stream and all working on caller-owned device buffers:
  *
  *   rf_schedule_compact  active-frame mask -> frame / token index lists
- *   rf_project           Eq. 3 for skipped frames, copy for active frames
+ *   rf_project           Eq. 3 for skipped frames' latents, copy for active frames
+ *   rf_project_kv        Eq. 3 for skipped frames' keys and values from the
+ *                        rolling cache of Appendix B.2; fresh rows shifted in
  *   rf_attn              active-query x full-sequence attention (bf16, tcgen05)
  *   rf_step              Euler update of the active frames
  *
@@ -245,9 +247,14 @@ int64_t rf_attn_workspace_bytes(int d);
  * up to 160 SMs), present on every GPU that loads the library until the
  * process exits.  The call allocates and frees nothing.
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current and caches it; make that
- *     first call before any stream capture.
- *   - Each call zeroes the array's counters on `stream` before the kernel runs.
+ *     (cudaGetSymbolAddress) with that device current and caches it for the
+ *     life of the process; make that first call before any stream capture.
+ *     cudaDeviceReset (or any other teardown of the device's primary context)
+ *     invalidates the cached address: do not call rf_attn_noalloc on a device
+ *     after resetting it.
+ *   - Argument errors (those rf_attn returns) are returned before anything is
+ *     enqueued.  Otherwise each call zeroes the array's counters on `stream`
+ *     before the kernel runs.
  *   - Every call on a device shares the one array, and it keeps the last call's
  *     contents: calls that overlap on the GPU (different streams, or several
  *     host threads) race on it and give wrong results.  Issue them in order on
@@ -314,16 +321,21 @@ rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double
 
 /*
  * rf_pipeline -- the step core fed from pinned host memory: one asynchronous denoising step
- * (Algorithm 2: rf_schedule_compact, rf_project, rf_attn, rf_step) per rf_pipeline_step,
- * with the step's inputs copied from the host and its results copied back, the copies of
- * neighbouring steps overlapped with the compute of the current one.  No paper passage: this
- * is the host side of serving the step core.
+ * (Algorithm 2: rf_schedule_compact, rf_project, rf_project_kv, rf_attn, rf_step) per
+ * rf_pipeline_step, with the step's inputs copied from the host and its results copied back,
+ * the copies of neighbouring steps overlapped with the compute of the current one.  The keys
+ * and values of skipped frames never cross the bus: they are the Eq. 3 projection of the
+ * device-resident rolling cache (Appendix B.2).  No paper passage: this is the host side of
+ * serving the step core.
  *
  * rf_pipeline_create allocates, on the current device, the plan, the two-slot latent store,
- * the index lists, an rf_attn workspace and `depth` buffer sets (Q, K, V, O bf16
- * [F*N][H][d]; velocity fp32 [F][E]; a latent-store snapshot fp32 [2][F][E]).
+ * the rolling key/value cache (bf16 [2][F][N][H*d] each), the index lists, an rf_attn
+ * workspace and `depth` buffer sets (Q, K, V, O bf16 [F*N][H][d]; velocity fp32 [F][E];
+ * snapshots of the latent store fp32 [2][F][E] and of the context fp32 [F][E]).
  *   h_mask, h_alpha, h_beta, h_dt, h_cur_slot  the plan, [S][F] as rf_plan_build writes it
  *   h_z2        fp32 [2][F][E] initial two-slot latent store
+ *   h_K0, h_V0  bf16 [F*N][H][d] initial keys and values: both cache slots of every frame
+ *               start with them (the cache's counterpart of both latent slots holding z0)
  *   depth       buffer sets, 2..8 (3 lets a heavy step's input copies run during the two
  *               steps before it)
  *   compute, h2d, d2h  three streams the pipeline enqueues on (all work of a step is
@@ -332,11 +344,12 @@ rf_status rf_keyframe_select(const double* h_G, int F, int M, double tau, double
  * d in {64, 128}; E % 4 == 0.
  *
  * rf_pipeline_step enqueues schedule step s (0 <= s < S) and returns:
- *   h_Q, h_K, h_V  pinned host bf16 [F*N][H][d] (rows contiguous); only the rows of the
- *               frames active at step s are read from h_Q
+ *   h_Q, h_K, h_V  pinned host bf16 [F*N][H][d] (rows contiguous): the fresh queries, keys
+ *               and values; only the rows of the frames active at step s are read
  *   h_v         pinned host fp32 [F][E] velocity of the step
  *   h_O         pinned host bf16 [F*N][H][d]: the active frames' rows are written
  *   h_z2        pinned host fp32 [2][F][E]: the latent store after the step
+ *   h_ctx       pinned host fp32 [F][E] (nullable): the step's Eq. 3 latent context
  *   softmax_scale  as for rf_attn
  * Host buffers of a step must stay valid and untouched until rf_pipeline_sync; the buffers
  * of `depth` consecutive steps may be in flight at once.  A step that returns an error may
@@ -352,11 +365,12 @@ typedef struct rf_pipeline rf_pipeline;
 rf_status rf_pipeline_create(int F, int N, int H, int d, int64_t E, int S,
                              const uint8_t* h_mask, const float* h_alpha, const float* h_beta,
                              const float* h_dt, const uint8_t* h_cur_slot, const float* h_z2,
-                             int depth, rf_stream_t compute, rf_stream_t h2d, rf_stream_t d2h,
+                             const void* h_K0, const void* h_V0, int depth,
+                             rf_stream_t compute, rf_stream_t h2d, rf_stream_t d2h,
                              rf_pipeline** out);
 rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, const void* h_K,
                            const void* h_V, const float* h_v, void* h_O, float* h_z2,
-                           float softmax_scale);
+                           float* h_ctx, float softmax_scale);
 rf_status rf_pipeline_sync(rf_pipeline* p, int32_t* h_status);
 rf_status rf_pipeline_bytes(const rf_pipeline* p, int64_t* h_steps, int64_t* h_h2d_bytes,
                             int64_t* h_d2h_bytes);

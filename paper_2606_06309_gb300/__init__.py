@@ -55,8 +55,8 @@ _SIG = {
                          _f32, _vp, _vp], _i32),
     "rf_step": ([_vp, _vp, _vp, _vp, _vp, _vp, _i32, _i64, _vp], _i32),
     "rf_pipeline_create": ([_i32, _i32, _i32, _i32, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
-                            _i32, _vp, _vp, _vp, ctypes.POINTER(_vp)], _i32),
-    "rf_pipeline_step": ([_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f32], _i32),
+                            _vp, _vp, _i32, _vp, _vp, _vp, ctypes.POINTER(_vp)], _i32),
+    "rf_pipeline_step": ([_vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _f32], _i32),
     "rf_pipeline_sync": ([_vp, _vp], _i32),
     "rf_pipeline_bytes": ([_vp, _vp, _vp, _vp], _i32),
     "rf_pipeline_destroy": ([_vp], None),
@@ -224,10 +224,12 @@ def rf_step(z2, cur_slot, v, dt, active, counts, F: int, E: int, stream=None):
         _stream(stream)))
 
 
-def rf_pipeline_create(F: int, N: int, H: int, d: int, E: int, plan: dict, z2, depth: int,
-                       compute, h2d, d2h) -> int:
-    """Host-fed step pipeline over the host plan (rf_plan_build's arrays) and an initial fp32
-    [2, F, E] latent store (host array or tensor); returns an opaque handle."""
+def rf_pipeline_create(F: int, N: int, H: int, d: int, E: int, plan: dict, z2, K0, V0,
+                       depth: int, compute, h2d, d2h) -> int:
+    """Host-fed step pipeline over the host plan (rf_plan_build's arrays), an initial fp32
+    [2, F, E] latent store (host array or tensor) and the initial keys and values K0, V0 (bf16
+    [F*N, H, d] contiguous host tensors) that both slots of the rolling cache start with;
+    returns an opaque handle."""
     # every array is bound to a name, so that none is freed before the call reads it
     mask = np.ascontiguousarray(plan["mask"], dtype=np.uint8)
     alpha = np.ascontiguousarray(plan["alpha"], dtype=np.float32)
@@ -235,17 +237,21 @@ def rf_pipeline_create(F: int, N: int, H: int, d: int, E: int, plan: dict, z2, d
     dt = np.ascontiguousarray(plan["dt"], dtype=np.float32)
     slot = np.ascontiguousarray(plan["cur_slot"], dtype=np.uint8)
     z = np.ascontiguousarray(np.asarray(z2.cpu() if hasattr(z2, "cpu") else z2), dtype=np.float32)
+    k0, v0 = (x.cpu().contiguous() if hasattr(x, "cpu") else np.ascontiguousarray(x)
+              for x in (K0, V0))
     S = mask.shape[0]
     out = _vp()
     _check("rf_pipeline_create", load().rf_pipeline_create(
         F, N, H, d, E, S, _ptr(mask), _ptr(alpha), _ptr(beta), _ptr(dt), _ptr(slot), _ptr(z),
-        depth, _stream(compute), _stream(h2d), _stream(d2h), ctypes.byref(out)))
+        _ptr(k0), _ptr(v0), depth, _stream(compute), _stream(h2d), _stream(d2h),
+        ctypes.byref(out)))
     return out.value
 
 
-def rf_pipeline_step(handle: int, s: int, hQ, hK, hV, hv, hO, hz2, softmax_scale: float):
+def rf_pipeline_step(handle: int, s: int, hQ, hK, hV, hv, hO, hz2, hctx,
+                     softmax_scale: float):
     _check("rf_pipeline_step", load().rf_pipeline_step(
-        handle, s, _ptr(hQ), _ptr(hK), _ptr(hV), _ptr(hv), _ptr(hO), _ptr(hz2),
+        handle, s, _ptr(hQ), _ptr(hK), _ptr(hV), _ptr(hv), _ptr(hO), _ptr(hz2), _ptr(hctx),
         float(softmax_scale)))
 
 

@@ -1224,11 +1224,13 @@ extern "C" int64_t rf_attn_workspace_bytes(int d) {
 }
 
 namespace {
-rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, const void* d_V,
-                    int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H, int d,
-                    const int32_t* d_active, const int32_t* d_counts, float softmax_scale,
-                    const uint8_t* d_block_mask, void* d_workspace, int64_t workspace_bytes_given,
-                    int32_t* d_status, rf_stream_t stream) {
+// Every host-checkable argument error of an attention call, before anything is enqueued.
+rf_status check_attn_args(const void* d_O, const void* d_Q, const void* d_K, const void* d_V,
+                          int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H,
+                          int d, const int32_t* d_active, const int32_t* d_counts,
+                          float softmax_scale, const uint8_t* d_block_mask,
+                          const void* d_workspace, int64_t workspace_bytes_given,
+                          DeviceInfo* di) {
   if (!d_O || !d_Q || !d_K || !d_V || !d_active || !d_counts) return RF_ERR_INVALID_ARG;
   if (F < 1 || N < 1 || H < 1 || H > 65535) return RF_ERR_INVALID_ARG;
   if (d != 64 && d != 128) return RF_ERR_UNSUPPORTED;
@@ -1248,9 +1250,23 @@ rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, c
     if (workspace_bytes_given < 0) return RF_ERR_INVALID_ARG;
     if (reinterpret_cast<uintptr_t>(d_workspace) & 255) return RF_ERR_MISALIGNED;
   }
+  if (rf_status st = current_device_info(di)) return st;
+  if (di->cc_major != 10 || di->cc_minor != 3) return fail(RF_ERR_UNSUPPORTED, "needs sm_103");
+  return RF_OK;
+}
+
+rf_status attn_impl(void* d_O, float* d_lse, const void* d_Q, const void* d_K, const void* d_V,
+                    int64_t qkv_row_stride, int64_t o_row_stride, int F, int N, int H, int d,
+                    const int32_t* d_active, const int32_t* d_counts, float softmax_scale,
+                    const uint8_t* d_block_mask, void* d_workspace, int64_t workspace_bytes_given,
+                    int32_t* d_status, rf_stream_t stream) {
   DeviceInfo di;
-  if (rf_status st = current_device_info(&di)) return st;
-  if (di.cc_major != 10 || di.cc_minor != 3) return fail(RF_ERR_UNSUPPORTED, "needs sm_103");
+  if (rf_status st = check_attn_args(d_O, d_Q, d_K, d_V, qkv_row_stride, o_row_stride, F, N, H,
+                                     d, d_active, d_counts, softmax_scale, d_block_mask,
+                                     d_workspace, workspace_bytes_given, &di))
+    return st;
+  const int64_t S_tok = static_cast<int64_t>(F) * N;
+  const int64_t Np = (static_cast<int64_t>(N) + 7) / 8 * 8;
 
   CUtensorMap mq, mq128, mk, mv;
   if (rf_status st = make_map(&mq, d_Q, d, H, static_cast<int>(S_tok), qkv_row_stride, 8)) return st;
@@ -1351,6 +1367,12 @@ extern "C" rf_status rf_attn_noalloc(void* d_O, float* d_lse, const void* d_Q, c
                                      int64_t o_row_stride, int F, int N, int H, int d,
                                      const int32_t* d_active, const int32_t* d_counts,
                                      float softmax_scale, int32_t* d_status, rf_stream_t stream) {
+  // Argument errors return before the counter reset below is enqueued.
+  DeviceInfo di;
+  if (rf_status st = check_attn_args(d_O, d_Q, d_K, d_V, qkv_row_stride, o_row_stride, F, N, H,
+                                     d, d_active, d_counts, softmax_scale, nullptr, nullptr, 0,
+                                     &di))
+    return st;
   int dev = 0;
   if (cudaError_t e = cudaGetDevice(&dev)) return fail(RF_ERR_CUDA, "cudaGetDevice", e);
   if (dev < 0 || dev >= 64) return fail(RF_ERR_UNSUPPORTED, "device ordinal >= 64");

@@ -2,11 +2,14 @@
 //
 // One asynchronous denoising step (Algorithm 2) per call, with its inputs copied from the host
 // and its results copied back, the copies of neighbouring steps overlapped with the compute of
-// the current one.  What a step reads: the query rows of the frames active at that step (the
-// attention reads no other query row), all keys and values, the velocity.  What it writes: the
-// active frames' rows of the attention output and the two-slot latent store.  `depth` device
-// buffer sets and three caller streams (compute, host->device, device->host) are ordered by
-// events; nothing synchronises the host until rf_pipeline_sync.
+// the current one.  What a step reads from the host: the query, key and value rows of the frames
+// active at that step (the fresh ones) and the velocity.  The keys and values of skipped frames
+// come from the device-resident rolling cache (Appendix B.2): rf_project_kv writes their Eq. 3
+// projection into the step's K/V buffers and shifts the fresh rows into the cache.  What a step
+// writes back: the active frames' rows of the attention output, the Eq. 3 latent context and
+// the two-slot latent store.  `depth` device buffer sets and three caller streams (compute,
+// host->device, device->host) are ordered by events; nothing synchronises the host until
+// rf_pipeline_sync.
 #include <cuda_runtime.h>
 
 #include <new>
@@ -34,6 +37,8 @@ struct rf_pipeline {
   // state
   float* z2 = nullptr;   // [2][F][E]
   float* ctx = nullptr;  // [F][E]
+  void* Kc = nullptr;    // rolling key/value cache, bf16 [2][F][N][H*d]
+  void* Vc = nullptr;
   int32_t* active = nullptr;
   int32_t* skipped = nullptr;
   int32_t* counts = nullptr;
@@ -44,6 +49,7 @@ struct rf_pipeline {
     void *Q, *K, *V, *O;
     float* v;
     float* z;
+    float* ctx;
     cudaEvent_t loaded, consumed, drained;
   };
   std::vector<Set> sets;
@@ -88,7 +94,7 @@ namespace {
 
 rf_status create(rf_pipeline* p, const uint8_t* h_mask, const float* h_alpha,
                  const float* h_beta, const float* h_dt, const uint8_t* h_cur_slot,
-                 const float* h_z2) {
+                 const float* h_z2, const void* h_K0, const void* h_V0) {
   const size_t SF = static_cast<size_t>(p->S) * p->F;
   const size_t FE = static_cast<size_t>(p->F) * p->E;
   void* v = nullptr;
@@ -103,6 +109,9 @@ rf_status create(rf_pipeline* p, const uint8_t* h_mask, const float* h_alpha,
   RF_TRY(alloc(p, &v, static_cast<size_t>(p->F) * 4)); p->skipped = static_cast<int32_t*>(v);
   RF_TRY(alloc(p, &v, 2 * 4)); p->counts = static_cast<int32_t*>(v);
   RF_TRY(alloc(p, &v, 4)); p->status = static_cast<int32_t*>(v);
+  const size_t qkv = static_cast<size_t>(p->S_tok) * p->row_bytes;
+  RF_TRY(alloc(p, &p->Kc, 2 * qkv));
+  RF_TRY(alloc(p, &p->Vc, 2 * qkv));
   p->ws_bytes = rf_attn_workspace_bytes(p->d);
   if (p->ws_bytes < 0) return fail(RF_ERR_CUDA, "rf_attn_workspace_bytes (rf_pipeline)");
   RF_TRY(alloc(p, &p->ws, static_cast<size_t>(p->ws_bytes)));
@@ -112,10 +121,17 @@ rf_status create(rf_pipeline* p, const uint8_t* h_mask, const float* h_alpha,
   CUDA_TRY(cudaMemcpy(p->dt, h_dt, SF * 4, cudaMemcpyHostToDevice), "plan upload");
   CUDA_TRY(cudaMemcpy(p->cur_slot, h_cur_slot, SF, cudaMemcpyHostToDevice), "plan upload");
   CUDA_TRY(cudaMemcpy(p->z2, h_z2, 2 * FE * 4, cudaMemcpyHostToDevice), "state upload");
+  // both cache slots of every frame start with the initial keys and values (the identity for
+  // a frame projected before its second update, as both latent slots start with z0)
+  for (int slot = 0; slot < 2; ++slot) {
+    CUDA_TRY(cudaMemcpy(static_cast<char*>(p->Kc) + slot * qkv, h_K0, qkv, cudaMemcpyHostToDevice),
+             "cache upload");
+    CUDA_TRY(cudaMemcpy(static_cast<char*>(p->Vc) + slot * qkv, h_V0, qkv, cudaMemcpyHostToDevice),
+             "cache upload");
+  }
   CUDA_TRY(cudaMemset(p->ws, 0, static_cast<size_t>(p->ws_bytes)), "workspace");
   CUDA_TRY(cudaMemset(p->status, 0, 4), "status");
   p->h_mask.assign(h_mask, h_mask + SF);
-  const size_t qkv = static_cast<size_t>(p->S_tok) * p->row_bytes;
   p->sets.resize(p->depth);
   for (rf_pipeline::Set& B : p->sets) {
     RF_TRY(alloc(p, &B.Q, qkv));
@@ -124,6 +140,7 @@ rf_status create(rf_pipeline* p, const uint8_t* h_mask, const float* h_alpha,
     RF_TRY(alloc(p, &B.O, qkv));
     RF_TRY(alloc(p, &v, FE * 4)); B.v = static_cast<float*>(v);
     RF_TRY(alloc(p, &v, 2 * FE * 4)); B.z = static_cast<float*>(v);
+    RF_TRY(alloc(p, &v, FE * 4)); B.ctx = static_cast<float*>(v);
     RF_TRY(event(p, &B.loaded));
     RF_TRY(event(p, &B.consumed));
     RF_TRY(event(p, &B.drained));
@@ -136,12 +153,14 @@ rf_status create(rf_pipeline* p, const uint8_t* h_mask, const float* h_alpha,
 extern "C" rf_status rf_pipeline_create(int F, int N, int H, int d, int64_t E, int S,
                                         const uint8_t* h_mask, const float* h_alpha,
                                         const float* h_beta, const float* h_dt,
-                                        const uint8_t* h_cur_slot, const float* h_z2, int depth,
+                                        const uint8_t* h_cur_slot, const float* h_z2,
+                                        const void* h_K0, const void* h_V0, int depth,
                                         rf_stream_t compute, rf_stream_t h2d, rf_stream_t d2h,
                                         rf_pipeline** out) {
   if (!out) return RF_ERR_INVALID_ARG;
   *out = nullptr;
-  if (!h_mask || !h_alpha || !h_beta || !h_dt || !h_cur_slot || !h_z2) return RF_ERR_INVALID_ARG;
+  if (!h_mask || !h_alpha || !h_beta || !h_dt || !h_cur_slot || !h_z2 || !h_K0 || !h_V0)
+    return RF_ERR_INVALID_ARG;
   if (F < 1 || F > 65535 || N < 1 || H < 1 || S < 1 || E < 4 || depth < 2 || depth > 8)
     return RF_ERR_INVALID_ARG;
   if (d != 64 && d != 128) return RF_ERR_UNSUPPORTED;
@@ -160,7 +179,7 @@ extern "C" rf_status rf_pipeline_create(int F, int N, int H, int d, int64_t E, i
   p->compute = reinterpret_cast<cudaStream_t>(compute);
   p->h2d = reinterpret_cast<cudaStream_t>(h2d);
   p->d2h = reinterpret_cast<cudaStream_t>(d2h);
-  if (rf_status st = create(p, h_mask, h_alpha, h_beta, h_dt, h_cur_slot, h_z2)) {
+  if (rf_status st = create(p, h_mask, h_alpha, h_beta, h_dt, h_cur_slot, h_z2, h_K0, h_V0)) {
     release(p);
     return st;
   }
@@ -170,7 +189,7 @@ extern "C" rf_status rf_pipeline_create(int F, int N, int H, int d, int64_t E, i
 
 extern "C" rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, const void* h_K,
                                       const void* h_V, const float* h_v, void* h_O, float* h_z2,
-                                      float softmax_scale) {
+                                      float* h_ctx, float softmax_scale) {
   if (!p || !h_Q || !h_K || !h_V || !h_v || !h_O || !h_z2) return RF_ERR_INVALID_ARG;
   if (s < 0 || s >= p->S) return RF_ERR_INVALID_ARG;
   const int F = p->F;
@@ -193,17 +212,18 @@ extern "C" rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, co
   }
   int64_t active_bytes = 0;
   // host -> device
+  // host -> device: the fresh Q, K and V rows of the active frames, and the velocity
   if (!first_use) CUDA_TRY(cudaStreamWaitEvent(p->h2d, B.consumed, 0), "rf_pipeline h2d wait");
   for (const auto& r : runs) {
     const int64_t off = r.first * frame_bytes, n = (r.second - r.first) * frame_bytes;
-    CUDA_TRY(cudaMemcpyAsync(static_cast<char*>(B.Q) + off, static_cast<const char*>(h_Q) + off,
-                             n, cudaMemcpyHostToDevice, p->h2d),
-             "rf_pipeline Q copy");
+    const std::pair<void*, const void*> qkv[3] = {{B.Q, h_Q}, {B.K, h_K}, {B.V, h_V}};
+    for (const auto& x : qkv)
+      CUDA_TRY(cudaMemcpyAsync(static_cast<char*>(x.first) + off,
+                               static_cast<const char*>(x.second) + off, n,
+                               cudaMemcpyHostToDevice, p->h2d),
+               "rf_pipeline Q/K/V copy");
     active_bytes += n;
   }
-  const int64_t kv = p->S_tok * p->row_bytes;
-  CUDA_TRY(cudaMemcpyAsync(B.K, h_K, kv, cudaMemcpyHostToDevice, p->h2d), "rf_pipeline K copy");
-  CUDA_TRY(cudaMemcpyAsync(B.V, h_V, kv, cudaMemcpyHostToDevice, p->h2d), "rf_pipeline V copy");
   CUDA_TRY(cudaMemcpyAsync(B.v, h_v, FE4, cudaMemcpyHostToDevice, p->h2d), "rf_pipeline v copy");
   CUDA_TRY(cudaEventRecord(B.loaded, p->h2d), "rf_pipeline event");
   // the step core on the compute stream
@@ -215,11 +235,17 @@ extern "C" rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, co
   RF_TRY(rf_schedule_compact(p->mask + o, F, p->N, p->active, p->skipped, nullptr, p->counts, cs));
   RF_TRY(rf_project(p->ctx, p->z2, p->cur_slot + o, p->alpha + o, p->beta + o, F, p->E, cs));
   const int64_t hd = static_cast<int64_t>(p->H) * p->d;
+  // skipped frames' keys and values: Eq. 3 over the cache; active frames' fresh rows shifted in
+  RF_TRY(rf_project_kv(B.K, B.V, hd, p->Kc, p->Vc, p->cur_slot + o, p->alpha + o, p->beta + o,
+                       p->active, p->skipped, p->counts, F, p->N, static_cast<int>(hd), cs));
   RF_TRY(rf_attn(B.O, nullptr, B.Q, B.K, B.V, hd, hd, F, p->N, p->H, p->d, p->active, p->counts,
                  softmax_scale, p->ws, p->ws_bytes, p->status, cs));
   RF_TRY(rf_step(p->z2, p->cur_slot + o, B.v, p->dt + o, p->active, p->counts, F, p->E, cs));
   CUDA_TRY(cudaMemcpyAsync(B.z, p->z2, 2 * FE4, cudaMemcpyDeviceToDevice, p->compute),
            "rf_pipeline state snapshot");
+  if (h_ctx)
+    CUDA_TRY(cudaMemcpyAsync(B.ctx, p->ctx, FE4, cudaMemcpyDeviceToDevice, p->compute),
+             "rf_pipeline context snapshot");
   CUDA_TRY(cudaEventRecord(B.consumed, p->compute), "rf_pipeline event");
   // device -> host
   CUDA_TRY(cudaStreamWaitEvent(p->d2h, B.consumed, 0), "rf_pipeline d2h wait");
@@ -231,10 +257,13 @@ extern "C" rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, co
   }
   CUDA_TRY(cudaMemcpyAsync(h_z2, B.z, 2 * FE4, cudaMemcpyDeviceToHost, p->d2h),
            "rf_pipeline state copy");
+  if (h_ctx)
+    CUDA_TRY(cudaMemcpyAsync(h_ctx, B.ctx, FE4, cudaMemcpyDeviceToHost, p->d2h),
+             "rf_pipeline context copy");
   CUDA_TRY(cudaEventRecord(B.drained, p->d2h), "rf_pipeline event");
   ++p->steps;
-  p->h2d_bytes += active_bytes + 2 * kv + static_cast<int64_t>(FE4);
-  p->d2h_bytes += active_bytes + 2 * static_cast<int64_t>(FE4);
+  p->h2d_bytes += 3 * active_bytes + static_cast<int64_t>(FE4);
+  p->d2h_bytes += active_bytes + (h_ctx ? 3 : 2) * static_cast<int64_t>(FE4);
   return RF_OK;
 }
 

@@ -1,14 +1,17 @@
-"""Device state and the four-call sequence of one asynchronous denoising step.
+"""Device state and the five-call sequence of one asynchronous denoising step.
 
 One step s of Algorithm 2 on the device, all on one CUDA stream, no host
 synchronisation:
 
   1. rf_schedule_compact(mask[s])  -> active / skipped frame lists, token list, counts
-  2. rf_project(...)               -> full-sequence context at sigma_s (Eq. 3)
-  3. rf_attn(...)                  -> active queries x all keys (Q/K/V supplied by the
-                                      caller; the DiT projections that would produce them
-                                      from the context are outside this library)
-  4. rf_step(...)                  -> Euler update of the active frames (two-slot store)
+  2. rf_project(...)               -> full-sequence latent context at sigma_s (Eq. 3)
+  3. rf_project_kv(...)            -> keys and values of the skipped frames: Eq. 3 over the
+                                      rolling cache of Appendix B.2; the active frames' fresh
+                                      rows shifted into the cache
+  4. rf_attn(...)                  -> active queries x all keys (the active frames' Q/K/V
+                                      rows supplied by the caller; the DiT projections that
+                                      would produce them are outside this library)
+  5. rf_step(...)                  -> Euler update of the active frames (two-slot store)
 
 The plan (masks, Eq. 3 weights, step sizes, slot bits) comes from the host
 planner rf_plan_build and is uploaded once.  PyTorch only allocates memory.
@@ -22,7 +25,7 @@ import torch
 
 from . import (rf_attn, rf_attn_workspace_bytes, rf_pipeline_bytes, rf_pipeline_create,
                rf_pipeline_destroy, rf_pipeline_step, rf_pipeline_sync, rf_plan_build, rf_project,
-               rf_schedule_compact, rf_step)
+               rf_project_kv, rf_schedule_compact, rf_step)
 
 
 @dataclass
@@ -42,10 +45,14 @@ def upload_plan(F, S, is_key, stride, T_w, device, sigma=None) -> Plan:
 
 
 class StepCore:
-    """Buffers for F frames of N tokens, E latent elements per frame, H heads of dim d."""
+    """Buffers for F frames of N tokens, E latent elements per frame, H heads of dim d.
+
+    With kv_cache (the default) the step core holds the rolling key/value cache (bf16
+    [2, F, N, H*d] each) and run() fills the skipped frames' rows of K and V from it before
+    the attention; set_kv_cache() gives the cache its initial contents."""
 
     def __init__(self, F: int, N: int, E: int, H: int, d: int, plan: Plan, device="cuda",
-                 token_list: bool = True, split_kv: bool = True):
+                 token_list: bool = True, split_kv: bool = True, kv_cache: bool = True):
         self.F, self.N, self.E, self.H, self.d = F, N, E, H, d
         self.plan = plan
         dev = torch.device(device)
@@ -56,6 +63,10 @@ class StepCore:
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.z2 = torch.zeros(2, F, E, dtype=torch.float32, device=dev)
         self.ctx = torch.zeros(F, E, dtype=torch.float32, device=dev)
+        self.Kc = self.Vc = None
+        if kv_cache:
+            self.Kc = torch.zeros(2, F, N, H * d, dtype=torch.bfloat16, device=dev)
+            self.Vc = torch.zeros_like(self.Kc)
         # split-KV workspace for rf_attn: zero-filled once, left zeroed by every call
         self.workspace = None
         if split_kv:
@@ -65,6 +76,15 @@ class StepCore:
     def set_state(self, z0: torch.Tensor):
         self.z2[0].copy_(z0)
         self.z2[1].copy_(z0)
+
+    def set_kv_cache(self, K0: torch.Tensor, V0: torch.Tensor):
+        """Both cache slots of every frame hold the keys and values K0, V0 ([F*N, H, d]): a frame
+        projected before its second update gets them back (alpha weights two equal states)."""
+        D = self.H * self.d
+        for c, X in ((self.Kc, K0), (self.Vc, V0)):
+            x = X.reshape(self.F, self.N, D)
+            c[0].copy_(x)
+            c[1].copy_(x)
 
     def current(self, s: int) -> torch.Tensor:
         """State of every frame when step s begins (s = S: the final state)."""
@@ -84,6 +104,11 @@ class StepCore:
         rf_project(self.ctx, self.z2, self.plan.cur_slot[s], self.plan.alpha[s],
                    self.plan.beta[s], self.F, self.E, stream)
 
+    def project_kv(self, s: int, K, V, stream=None):
+        rf_project_kv(K, V, K.stride(0), self.Kc, self.Vc, self.plan.cur_slot[s],
+                      self.plan.alpha[s], self.plan.beta[s], self.active, self.skipped,
+                      self.counts, self.F, self.N, self.H * self.d, stream)
+
     def attn(self, O, Q, K, V, scale: float, lse: Optional[torch.Tensor] = None, stream=None):
         rf_attn(O, lse, Q, K, V, Q.stride(0), O.stride(0), self.F, self.N, self.H, self.d,
                 self.active, self.counts, scale, self.workspace, self.status, stream)
@@ -93,13 +118,21 @@ class StepCore:
                 self.F, self.E, stream)
 
     def run(self, s: int, v, O, Q, K, V, scale: float, lse=None, stream=None):
+        """Step s.  Q, K, V hold the active frames' fresh rows; with the cache, the skipped
+        frames' rows of K and V are overwritten with their projection before the attention."""
         self.compact(s, stream)
         self.project(s, stream)
+        if self.Kc is not None:
+            self.project_kv(s, K, V, stream)
         self.attn(O, Q, K, V, scale, lse, stream)
         self.step(s, v, stream)
 
+    @property
+    def launches_per_step(self) -> int:
+        return 5 if self.Kc is not None else 4
+
     def capture_trajectory(self, vels, O, Q, K, V, scale: float, steps=None):
-        """Record steps 0..S-1 (4 launches each) into one CUDA graph and return it.
+        """Record steps 0..S-1 (all launches of each) into one CUDA graph and return it.
 
         Nothing in the step core synchronises the host (counts stay on the device), so the
         whole trajectory replays with one launch.  Every call is made once eagerly first, so
@@ -120,21 +153,22 @@ class HostPipeline:
     """Step-core steps fed from pinned host memory, with the copies hidden behind compute.
 
     A thin wrapper of the library's native pipeline (``rf_pipeline_*``), which owns the plan,
-    the two-slot latent store and `depth` device buffer sets.  Each step copies host -> device
-    what it reads: the query rows of the frames active at that step (the attention reads no
-    other query row), all of K and V, and the velocity.  It copies device -> host what it
-    writes: the active frames' rows of the attention output and a snapshot of the latent
+    the two-slot latent store, the rolling key/value cache and `depth` device buffer sets.  Each
+    step copies host -> device what it reads: the fresh query, key and value rows of the frames
+    active at that step, and the velocity (the skipped frames' keys and values are projected
+    from the device-resident cache).  It copies device -> host what it writes: the active
+    frames' rows of the attention output, the latent context and a snapshot of the latent
     store.  Three streams (compute, host->device, device->host) are ordered by events, so the
     input copies of the next depth-1 steps and the read-back of earlier steps run during the
     compute of step k; nothing synchronises the host.  Three sets, not two: steps differ in
     cost (all frames active, then only the keyframes), and with two sets the inputs of a heavy
-    step could only be copied during the short light step before it (0.84 ms of copies against
-    0.5 ms of compute on 13 x 1560 tokens).
+    step could only be copied during the short light step before it.
 
-    The pipeline starts from `core`'s plan and current latent store; it does not change `core`.
+    The pipeline starts from `core`'s plan and current latent store, and from the initial keys
+    and values K0, V0 (host tensors); it does not change `core`.
     """
 
-    def __init__(self, core: StepCore, S_tok: int, device="cuda", depth: int = 3):
+    def __init__(self, core: StepCore, S_tok: int, K0, V0, device="cuda", depth: int = 3):
         dev = torch.device(device)
         self.core = core
         self.N = S_tok // core.F
@@ -144,14 +178,16 @@ class HostPipeline:
         self.d2h = torch.cuda.Stream(dev)
         torch.cuda.synchronize(dev)  # the core's latent store is read below
         self.handle = rf_pipeline_create(core.F, self.N, core.H, core.d, core.E, core.plan.host,
-                                         core.z2, depth, self.compute, self.h2d, self.d2h)
+                                         core.z2, K0, V0, depth, self.compute, self.h2d,
+                                         self.d2h)
         self._marks = []  # (steps, h2d bytes, d2h bytes) after each step
 
-    def step(self, s: int, hQ, hK, hV, hv, hO, hz, scale: float):
+    def step(self, s: int, hQ, hK, hV, hv, hO, hz, scale: float, hctx=None):
         """Enqueue schedule step s: inputs from pinned host tensors hQ, hK, hV (bf16
-        [S_tok, H, d], contiguous rows) and hv (fp32 [F, E]); results into pinned hO (bf16; the
-        active frames' rows) and hz (fp32 [2, F, E]).  Returns immediately."""
-        rf_pipeline_step(self.handle, s, hQ, hK, hV, hv, hO, hz, scale)
+        [S_tok, H, d], contiguous rows; the active frames' rows are read) and hv (fp32 [F, E]);
+        results into pinned hO (bf16; the active frames' rows), hz (fp32 [2, F, E]) and, if
+        given, hctx (fp32 [F, E], the Eq. 3 context).  Returns immediately."""
+        rf_pipeline_step(self.handle, s, hQ, hK, hV, hv, hO, hz, hctx, scale)
         self._marks.append(rf_pipeline_bytes(self.handle))
 
     def sync(self) -> int:

@@ -10,12 +10,12 @@ down over thousands of keys, but not on rows dominated by a few keys),
 accumulates in fp32 and evaluates exp2 with the hardware approximation
 (relative ~2^-22).
 
-The max-abs bound is read relative to the output's magnitude where |O| > 1:
-|g - o| <= 2e-2 * max(1, |o|).  bf16 keeps 8 significant bits, so an output of
-4.25 is stored to within half an ulp of 0.0156 and one of 8 or more only to
-within 0.031: an absolute 2e-2 cannot hold there for any bf16 result.  Rows
-with |O| of several units occur where a few large keys dominate (the 21 x 3600
-workload's tokens with std 2).
+The max-abs bound is 2e-2 plus the rounding of the stored output itself:
+|g - o| <= 2e-2 + ulp_bf16(|o|) / 2 where |o| >= 1, and exactly 2e-2 below 1.
+bf16 keeps 8 significant bits, so the nearest bf16 value to an output in
+[2^e, 2^(e+1)) can be 2^(e-8) away from it: 0.0078 in [2, 4), 0.0156 in [4, 8).
+Outputs of that size occur where a few large keys dominate a row (the tokens
+with std 2 of the 21 x 3600-token workload).  Nothing else is scaled with |o|.
 """
 import numpy as np
 
@@ -25,6 +25,19 @@ REL_FRO = 1e-2
 LSE_ABS = 1e-3
 
 
+def half_ulp_bf16(x):
+    """Half the spacing of bf16 values at |x| (8 significant bits): 2^(floor(log2|x|) - 8)."""
+    a = np.abs(np.asarray(x, dtype=np.float64))
+    e = np.floor(np.log2(np.maximum(a, np.finfo(np.float64).tiny)))
+    return np.exp2(e - 8.0)
+
+
+def max_abs_bound(o_ref):
+    """Per-element max-abs bound: 2e-2, plus half a bf16 ulp of |o| where |o| >= 1."""
+    r = np.abs(np.asarray(o_ref, dtype=np.float64))
+    return MAX_ABS + np.where(r >= 1.0, half_ulp_bf16(r), 0.0)
+
+
 def compare(o_gpu, o_ref, lse_gpu=None, lse_ref=None, label=""):
     g = np.asarray(o_gpu, dtype=np.float64)
     r = np.asarray(o_ref, dtype=np.float64)
@@ -32,14 +45,19 @@ def compare(o_gpu, o_ref, lse_gpu=None, lse_ref=None, label=""):
     assert np.isfinite(g).all(), f"{label}: non-finite output"
     err = np.abs(g - r)
     rel = np.linalg.norm(g - r) / max(np.linalg.norm(r), 1e-30)
-    ratio = err / (MAX_ABS * np.maximum(1.0, np.abs(r)))
+    ratio = err / max_abs_bound(r)
     i = np.unravel_index(np.argmax(ratio), ratio.shape)
-    msg = (f"{label}: max {err.max():.3e}, worst against the bound {ratio[i]:.2f} "
-           f"(gpu {g[i]:.5f}, oracle {r[i]:.5f}) mean {err.mean():.3e} relF {rel:.3e}")
+    msg = (f"{label}: max-abs {err.max():.3e} (absolute bound {MAX_ABS:g}), worst against the "
+           f"per-element bound {ratio[i]:.2f} (gpu {g[i]:.5f}, oracle {r[i]:.5f}) "
+           f"mean {err.mean():.3e} relF {rel:.3e}")
     assert ratio.max() <= 1.0, msg
     assert err.mean() <= MEAN_ABS, msg
     assert rel <= REL_FRO, msg
+    out = {"max": float(err.max()), "worst_ratio": float(ratio.max()),
+           "mean": float(err.mean()), "rel": float(rel)}
     if lse_gpu is not None:
         dl = np.abs(np.asarray(lse_gpu, np.float64) - np.asarray(lse_ref, np.float64)).max()
         assert dl <= LSE_ABS, f"{label}: lse {dl:.3e}"
-    return {"max": float(err.max()), "mean": float(err.mean()), "rel": float(rel)}
+        out["lse"] = float(dl)
+    print(msg)
+    return out

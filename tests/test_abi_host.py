@@ -118,13 +118,17 @@ def test_pipeline_rejects_bad_args_on_host(rf):
     lib = rf.load()
     P = 256
     out = ctypes.c_void_p(12345)
-    pa = [4, 8, 2, 128, 64, 3, P, P, P, P, P, P, 3, None, None, None, ctypes.byref(out)]
+    pa = [4, 8, 2, 128, 64, 3, P, P, P, P, P, P, P, P, 3, None, None, None, ctypes.byref(out)]
     bad = list(pa)
-    bad[16] = None
+    bad[18] = None
     assert lib.rf_pipeline_create(*bad) == 1                          # no handle to write
     bad = list(pa)
     bad[6] = None
     assert lib.rf_pipeline_create(*bad) == 1 and out.value is None    # null plan; handle cleared
+    for i in (12, 13):
+        bad = list(pa)
+        bad[i] = None
+        assert lib.rf_pipeline_create(*bad) == 1                      # no initial keys/values
     bad = list(pa)
     bad[3] = 96
     assert lib.rf_pipeline_create(*bad) == 2                          # d = 96 unsupported
@@ -133,9 +137,9 @@ def test_pipeline_rejects_bad_args_on_host(rf):
     assert lib.rf_pipeline_create(*bad) == 3                          # E % 4 != 0
     for depth in (1, 9):
         bad = list(pa)
-        bad[12] = depth
+        bad[14] = depth
         assert lib.rf_pipeline_create(*bad) == 1                      # depth outside 2..8
-    assert lib.rf_pipeline_step(None, 0, P, P, P, P, P, P, 0.1) == 1
+    assert lib.rf_pipeline_step(None, 0, P, P, P, P, P, P, None, 0.1) == 1
     assert lib.rf_pipeline_sync(None, None) == 1
     assert lib.rf_pipeline_bytes(None, None, None, None) == 1
     lib.rf_pipeline_destroy(None)                                     # a no-op
@@ -146,14 +150,15 @@ def test_python_binding_raises_with_status(rf):
     the library's last-error text in the message (host-side checks; no GPU is touched)."""
     plan = rf.rf_plan_build(3, 4, [1, 0, 1], [2] * 4, 0)
     z2 = np.zeros((2, 3, 16), np.float32)
+    kv = np.zeros((24, 2, 64), np.uint16)                               # bf16 bits
     with pytest.raises(rf.RFError) as e:
-        rf.rf_pipeline_create(3, 8, 2, 96, 16, plan, z2, 3, 0, 0, 0)   # head dim 96
+        rf.rf_pipeline_create(3, 8, 2, 96, 16, plan, z2, kv, kv, 3, 0, 0, 0)   # head dim 96
     assert e.value.status == 2 and "rf_pipeline_create" in str(e.value)
     with pytest.raises(rf.RFError) as e:
-        rf.rf_pipeline_create(3, 8, 2, 64, 18, plan, z2, 3, 0, 0, 0)   # E % 4 != 0
+        rf.rf_pipeline_create(3, 8, 2, 64, 18, plan, z2, kv, kv, 3, 0, 0, 0)   # E % 4 != 0
     assert e.value.status == 3
     with pytest.raises(rf.RFError) as e:
-        rf.rf_pipeline_create(3, 8, 2, 64, 16, plan, z2, 1, 0, 0, 0)   # depth 1
+        rf.rf_pipeline_create(3, 8, 2, 64, 16, plan, z2, kv, kv, 1, 0, 0, 0)   # depth 1
     assert e.value.status == 1
     assert rf.rf_status_str(2) and rf.rf_status_str(99)
 

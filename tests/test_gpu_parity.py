@@ -29,7 +29,7 @@ def _plan(rf, w):
 # ---------------------------------------------------------------------------
 def _masks():
     out = []
-    for name in ("tiny", "small", "mid", "long"):
+    for name in ("tiny", "small", "mid", "large", "long"):
         w = wl.get(name)
         p = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
         for row in np.unique(p["mask"], axis=0):
@@ -369,8 +369,46 @@ def test_attn_small_every_row_of_two_heads(cuda_lib, s):
 # ---------------------------------------------------------------------------
 # Whole trajectory: compaction + projection + attention + Euler step, S steps
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("name", ["tiny", "small"])
+def _path_magnitude(z0, vels, plan):
+    """Per step s and element, M_s = |z0| + sum of |dt * v| over the frame's updates before s:
+    a bound on |z_start|, |z_end| and every partial sum that produced them, hence on the terms
+    of every fp32 operation behind the state and the context at step s."""
+    M = np.abs(oracle.to_f64(z0))
+    out = []
+    for s in range(plan["mask"].shape[0]):
+        out.append(M.copy())
+        act = plan["mask"][s].astype(bool)
+        M[act] += np.abs(plan["dt"][s][act])[:, None] * np.abs(oracle.to_f64(vels[s])[act])
+    out.append(M)
+    return out
+
+
+def _fresh_kv(K0, V0, s):
+    """The keys and values the model would compute for step s: K0 and V0 scaled by
+    1 + 0.03 s (distinct every step, rounded to bf16)."""
+    c = 1.0 + 0.03 * s
+    return (K0.float() * c).to(torch.bfloat16), (V0.float() * c).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("name", ["tiny", "small", "mid", "large", "long"])
 def test_trajectory_matches_oracle_sampler(cuda_lib, name):
+    """Algorithm 2's whole S-step loop through the library, all five calls of every step
+    (compaction, Eq. 3 on the latents, Eq. 3 on the rolling key/value cache, attention, Euler
+    update on the two-slot store), against the oracle run step by step alongside:
+
+    * the latent context at every step and the final latent, element by element, each
+      element's error measured against the magnitude of the terms that produced it (the path
+      magnitude M: |z0| plus every |dt * v| the frame took), as the single-call tests measure
+      against |beta * prev| + |alpha * cur| and |z| + |dt * v|; after at most 50 fp32
+      roundings per element it is below 4e-6 of M;
+    * the keys and values attention reads at every step (two heads; elements are independent):
+      skipped frames' rows within bf16 rounding of the oracle's cache projection, active
+      frames' rows the fresh ones, and the cache itself bit for bit at the end;
+    * the attention output of sampled active rows of those heads at several steps, against
+      the oracle's attention over its own (unrounded) projected keys and values.
+
+    The progressive strides (1 -> 4, 1 -> 6) change alpha, dt and the slot bits from one
+    segment to the next, which only the whole loop exercises."""
     from paper_2606_06309_gb300.stepcore import StepCore, upload_plan
     w = wl.get(name)
     plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, DEV)
@@ -378,20 +416,75 @@ def test_trajectory_matches_oracle_sampler(cuda_lib, name):
     core = StepCore(w.F, w.N, E, w.H, w.d, plan, DEV)
     z0 = wl.latents(w)
     core.set_state(z0.to(DEV))
-    Q, K, V = wl.qkv(w, device=DEV)
+    Q, K0, V0 = wl.qkv(w, device=DEV)
+    core.set_kv_cache(K0, V0)
+    K, V = K0.clone(), V0.clone()
     O = torch.zeros_like(Q)
     vels = [wl.velocity(w, s) for s in range(w.S)]
     oplan = oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)
     zT_ref, ctx_ref = oracle.sampler(z0, vels, oplan)
+    mags = _path_magnitude(z0, vels, oplan)
+
+    heads = [0, w.H - 1] if w.H > 1 else [0]
+    hidx = torch.tensor(heads, device=DEV)
+
+    def heads_of(X):  # [S_tok, H, d] -> fp64 [F, N, len(heads) * d]
+        return oracle.to_f64(X.index_select(1, hidx)).reshape(w.F, w.N, -1)
+
+    cK = np.stack([heads_of(K0)] * 2)
+    cV = np.stack([heads_of(V0)] * 2)
+    Qh = oracle.to_f64(Q.index_select(1, hidx))
+    skip_steps = [s for s in range(w.S) if 0 < oplan["mask"][s].sum() < w.F]
+    attn_steps = set(range(w.S)) if w.S_tok * w.H <= 300_000 else \
+        {0, skip_steps[0], skip_steps[len(skip_steps) // 2], skip_steps[-1]}
+    rng = np.random.default_rng(w.seed)
+    worst = 0.0
     for s in range(w.S):
+        Kf, Vf = _fresh_kv(K0, V0, s)
+        K.copy_(Kf)
+        V.copy_(Vf)
         core.run(s, vels[s].to(DEV), O, Q, K, V, w.softmax_scale)
         ctx = core.ctx.cpu().double().numpy()
-        err = np.abs(ctx - ctx_ref[s]).max() / max(np.abs(ctx_ref[s]).max(), 1.0)
+        err = _rel_err(ctx, ctx_ref[s], mags[s])
+        worst = max(worst, err)
         assert err <= 1e-5, (s, err)
+        # keys and values the attention read at step s
+        mask = oplan["mask"][s]
+        sl, al = oplan["cur_slot"][s], oplan["alpha"][s]
+        sk = mask == 0
+        proj = {}
+        for X, Xf, c, lab in ((K, Kf, cK, "K"), (V, Vf, cV, "V")):
+            fresh = heads_of(Xf)
+            want, c_new = oracle.project_kv_cache(fresh, c, sl, al, mask)
+            proj[lab] = want
+            got = heads_of(X)
+            if sk.any():
+                f_idx = np.flatnonzero(sk)
+                terms = (np.abs(1.0 - al[sk])[:, None, None] * np.abs(c[1 - sl[sk], f_idx])
+                         + np.abs(al[sk])[:, None, None] * np.abs(c[sl[sk], f_idx]))
+                assert (np.abs(got[sk] - want[sk]) <= 2.0 ** -8 * terms + 1e-30).all(), (s, lab)
+            np.testing.assert_array_equal(got[~sk], fresh[~sk])
+            c[...] = c_new
+        if s in attn_steps:
+            act = np.flatnonzero(mask)
+            rows = {int(f * w.N + p) for f in act for p in (0, w.N - 1)}
+            all_rows = np.array(_active_rows(mask, w.N))
+            rows.update(rng.choice(all_rows, size=min(64, len(all_rows)), replace=False).tolist())
+            rows = sorted(rows)
+            shape = (w.S_tok, len(heads), w.d)
+            Oref, _ = oracle.attention(Qh, proj["K"].reshape(shape), proj["V"].reshape(shape),
+                                       rows, w.softmax_scale)
+            compare(O.index_select(1, hidx).cpu().float().numpy()[rows], Oref,
+                    label=f"{name} step {s} attention over projected K/V")
     got = core.current(w.S).cpu().double().numpy()
-    err = np.abs(got - zT_ref).max() / max(np.abs(zT_ref).max(), 1.0)
+    err = _rel_err(got, zT_ref, mags[w.S])
     assert err <= 1e-5, err
+    for Xc, c in ((core.Kc, cK), (core.Vc, cV)):
+        g = oracle.to_f64(Xc.view(2, w.F, w.N, w.H, w.d).index_select(3, hidx))
+        np.testing.assert_array_equal(g.reshape(c.shape), c)
     assert core.status.item() == 0
+    print(f"{name}: worst context error {worst:.2e}, final latent {err:.2e} (of the path "
+          f"magnitude)")
 
 
 @pytest.mark.parametrize("F,N,H,d,mask", [
@@ -421,56 +514,78 @@ def test_attn_split_and_unsplit_agree_with_oracle(cuda_lib, F, N, H, d, mask):
     assert (O1.float() - O2.float()).abs().max().item() < 1e-2
 
 
+def _pipeline_against_device_path(F, N, H, d, E, plan_args, Q, K0, V0, vel, z0, scale, nsteps,
+                                  depth):
+    """The same steps on device-resident inputs (StepCore, fresh K/V rows written before each
+    step) and through the native host-fed pipeline (fresh rows copied from pinned host
+    memory, skipped frames' keys/values projected from its own device cache): O of the active
+    rows, the latent store and the context must be identical.  Returns the pipeline's byte
+    counts per step and the masks."""
+    from paper_2606_06309_gb300.stepcore import HostPipeline, StepCore, upload_plan
+
+    def fresh():
+        c = StepCore(F, N, E, H, d, upload_plan(F, *plan_args, DEV), DEV)
+        c.set_state(z0.to(DEV))
+        c.set_kv_cache(K0, V0)
+        return c
+
+    kv = [_fresh_kv(K0, V0, s) for s in range(nsteps)]
+    ref = fresh()
+    O = torch.zeros_like(Q)
+    K, V = K0.clone(), V0.clone()
+    outs = []
+    for s in range(nsteps):
+        K.copy_(kv[s][0])
+        V.copy_(kv[s][1])
+        ref.run(s, vel[s].to(DEV), O, Q, K, V, scale)
+        outs.append((O.cpu().clone(), ref.z2.cpu().clone(), ref.ctx.cpu().clone()))
+    assert ref.status.item() == 0
+
+    core = fresh()
+    pipe = HostPipeline(core, F * N, K0.cpu(), V0.cpu(), DEV, depth=depth)
+    hQ = Q.cpu().pin_memory()
+    hK = [k.cpu().pin_memory() for k, _ in kv]
+    hV = [v.cpu().pin_memory() for _, v in kv]
+    hv = [v.cpu().pin_memory() for v in vel[:nsteps]]
+    hO = [torch.zeros(Q.shape, dtype=Q.dtype).pin_memory() for _ in range(nsteps)]
+    hz = [torch.zeros(core.z2.shape).pin_memory() for _ in range(nsteps)]
+    hc = [torch.zeros(core.ctx.shape).pin_memory() for _ in range(nsteps)]
+    for s in range(nsteps):
+        pipe.step(s, hQ, hK[s], hV[s], hv[s], hO[s], hz[s], scale, hctx=hc[s])
+    assert pipe.sync() == 0
+    masks = ref.plan.host["mask"]
+    for s in range(nsteps):
+        act = np.array(_active_rows(masks[s], N))
+        assert torch.equal(hO[s][act], outs[s][0][act]), s
+        assert torch.equal(hz[s], outs[s][1]), s
+        assert torch.equal(hc[s], outs[s][2]), s
+        skipped = np.setdiff1d(np.arange(F * N), act)
+        assert (hO[s][skipped] == 0).all(), s      # rows no step writes are not copied back
+    nbytes = pipe.bytes_per_step()
+    pipe.close()
+    pipe.close()                                    # closing twice is harmless
+    return nbytes, masks
+
+
 @pytest.mark.parametrize("name,depth", [("tiny", 2), ("tiny", 5), ("small", 3)])
 def test_host_pipeline_matches_device_path(cuda_lib, name, depth):
     """The native host-fed pipeline (inputs from pinned host memory, copies overlapped with
-    compute, `depth` device buffer sets) gives exactly the outputs of the same steps run on
-    device-resident inputs, and counts the bytes it copies."""
-    from paper_2606_06309_gb300.stepcore import HostPipeline, StepCore, upload_plan
+    compute, `depth` device buffer sets, its own rolling key/value cache) gives exactly the
+    outputs of the same steps run on device-resident inputs, and counts the bytes it copies."""
     w = wl.get(name)
     E = w.N * w.C
-    Q, K, V = wl.qkv(w, device=DEV)
+    Q, K0, V0 = wl.qkv(w, device=DEV)
     vel = [wl.velocity(w, s) for s in range(w.S)]
-    z0 = wl.latents(w)
-
-    def fresh():
-        plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, DEV)
-        c = StepCore(w.F, w.N, E, w.H, w.d, plan, DEV)
-        c.set_state(z0.to(DEV))
-        return c
-
-    ref = fresh()
-    O = torch.zeros_like(Q)
-    outs = []
     nsteps = min(w.S, 6)
-    for s in range(nsteps):
-        ref.run(s, vel[s].to(DEV), O, Q, K, V, w.softmax_scale)
-        outs.append((O.cpu().clone(), ref.z2.cpu().clone()))
-
-    core = fresh()
-    pipe = HostPipeline(core, w.S_tok, DEV, depth=depth)
-    hQ, hK, hV = (x.cpu().pin_memory() for x in (Q, K, V))
-    hv = [v.pin_memory() for v in vel]
-    hO = [torch.zeros(Q.shape, dtype=Q.dtype).pin_memory() for _ in range(nsteps)]
-    hz = [torch.zeros(core.z2.shape).pin_memory() for _ in range(nsteps)]
-    for s in range(nsteps):
-        pipe.step(s, hQ, hK, hV, hv[s], hO[s], hz[s], w.softmax_scale)
-    assert pipe.sync() == 0
-    for s in range(nsteps):
-        act = np.array(_active_rows(oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)["mask"][s], w.N))
-        assert torch.equal(hO[s][act], outs[s][0][act]), s
-        assert torch.equal(hz[s], outs[s][1]), s
-        skipped = np.setdiff1d(np.arange(w.S_tok), act)
-        assert (hO[s][skipped] == 0).all(), s      # rows no step writes are not copied back
-    # bytes: active Q rows, K, V and v in; active O rows and both latent slots out
+    (h2d, d2h), masks = _pipeline_against_device_path(
+        w.F, w.N, w.H, w.d, E, (w.S, w.is_key, w.stride, w.T_w), Q, K0, V0, vel,
+        wl.latents(w), w.softmax_scale, nsteps, depth)
+    # bytes: the active frames' Q, K and V rows and the velocity in; the active O rows, both
+    # latent slots and the context out
     row = w.H * w.d * 2
-    n_act = sum(len(_active_rows(oracle.schedule(w.F, w.S, w.is_key, w.stride, w.T_w)["mask"][s],
-                                 w.N)) for s in range(nsteps))
-    h2d, d2h = pipe.bytes_per_step()
-    assert h2d == round((n_act * row + nsteps * (2 * w.S_tok * row + w.F * E * 4)) / nsteps)
-    assert d2h == round((n_act * row + nsteps * 2 * w.F * E * 4) / nsteps)
-    pipe.close()
-    pipe.close()                                    # closing twice is harmless
+    n_act = sum(len(_active_rows(masks[s], w.N)) for s in range(nsteps))
+    assert h2d == round((3 * n_act * row + nsteps * w.F * E * 4) / nsteps)
+    assert d2h == round((n_act * row + nsteps * 3 * w.F * E * 4) / nsteps)
 
 
 @pytest.mark.parametrize("F,N,H,d,keys,depth", [
@@ -480,43 +595,15 @@ def test_host_pipeline_matches_device_path(cuda_lib, name, depth):
 ])
 def test_host_pipeline_ragged_shapes(cuda_lib, F, N, H, d, keys, depth):
     """The native pipeline on ragged shapes gives the device path's outputs bit for bit."""
-    from paper_2606_06309_gb300.stepcore import HostPipeline, StepCore, upload_plan
     S, E = 10, N * 16
     is_key = [1 if f in keys else 0 for f in range(F)]
     g = torch.Generator(device=DEV).manual_seed(F * 100 + N)
-    Q, K, V = (torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
-               for _ in range(3))
+    Q, K0, V0 = (torch.randn(F * N, H, d, generator=g, device=DEV).to(torch.bfloat16)
+                 for _ in range(3))
     vel = [torch.randn(F, E, generator=g, device=DEV) for _ in range(S)]
     z0 = torch.randn(F, E, generator=g, device=DEV)
-    scale = 1 / math.sqrt(d)
-
-    def fresh():
-        c = StepCore(F, N, E, H, d, upload_plan(F, S, is_key, [2] * S, 0, DEV), DEV)
-        c.set_state(z0)
-        return c
-
-    ref = fresh()
-    O = torch.zeros_like(Q)
-    outs = []
-    for s in range(S):
-        ref.run(s, vel[s], O, Q, K, V, scale)
-        outs.append((O.cpu().clone(), ref.z2.cpu().clone()))
-    assert ref.status.item() == 0
-    core = fresh()
-    pipe = HostPipeline(core, F * N, DEV, depth=depth)
-    hQ, hK, hV = (x.cpu().pin_memory() for x in (Q, K, V))
-    hv = [v.cpu().pin_memory() for v in vel]
-    hO = [torch.zeros(Q.shape, dtype=Q.dtype).pin_memory() for _ in range(S)]
-    hz = [torch.zeros(core.z2.shape).pin_memory() for _ in range(S)]
-    for s in range(S):
-        pipe.step(s, hQ, hK, hV, hv[s], hO[s], hz[s], scale)
-    assert pipe.sync() == 0
-    mask = oracle.schedule(F, S, is_key, [2] * S, 0)["mask"]
-    for s in range(S):
-        act = np.array(_active_rows(mask[s], N))
-        assert torch.equal(hO[s][act], outs[s][0][act]), s
-        assert torch.equal(hz[s], outs[s][1]), s
-    pipe.close()
+    _pipeline_against_device_path(F, N, H, d, E, (S, is_key, [2] * S, 0), Q, K0, V0, vel, z0,
+                                  1 / math.sqrt(d), S, depth)
 
 
 # ---------------------------------------------------------------------------
@@ -649,11 +736,13 @@ def test_keyframes_from_device_gram_match_oracle(cuda_lib):
 
 @pytest.mark.parametrize("name", ["tiny", "small"])
 def test_graph_replay_matches_eager(cuda_lib, name):
-    """A whole trajectory captured in one CUDA graph and replayed gives the eager results."""
+    """A whole trajectory captured in one CUDA graph and replayed gives the eager results:
+    the latent store, the attention output, the keys/values with their projected rows and the
+    rolling cache."""
     from paper_2606_06309_gb300.stepcore import StepCore, upload_plan
     w = wl.get(name)
     E = w.N * w.C
-    Q, K, V = wl.qkv(w, device=DEV)
+    Q, K0, V0 = wl.qkv(w, device=DEV)
     vels = [wl.velocity(w, s, device=DEV) for s in range(w.S)]
     z0 = wl.latents(w, device=DEV)
 
@@ -661,23 +750,31 @@ def test_graph_replay_matches_eager(cuda_lib, name):
         plan = upload_plan(w.F, w.S, w.is_key, w.stride, w.T_w, DEV)
         c = StepCore(w.F, w.N, E, w.H, w.d, plan, DEV)
         c.set_state(z0)
+        c.set_kv_cache(K0, V0)
         return c
 
     eager = fresh()
     O1 = torch.zeros_like(Q)
+    K1, V1 = K0.clone(), V0.clone()
     for s in range(w.S):
-        eager.run(s, vels[s], O1, Q, K, V, w.softmax_scale)
+        eager.run(s, vels[s], O1, Q, K1, V1, w.softmax_scale)
     torch.cuda.synchronize()
 
     cg = fresh()
     O2 = torch.zeros_like(Q)
-    g = cg.capture_trajectory(vels, O2, Q, K, V, w.softmax_scale)  # runs step 0 once eagerly
+    K2, V2 = K0.clone(), V0.clone()
+    g = cg.capture_trajectory(vels, O2, Q, K2, V2, w.softmax_scale)  # runs step 0 eagerly
     cg.set_state(z0)
+    cg.set_kv_cache(K0, V0)
+    K2.copy_(K0)
+    V2.copy_(V0)
     O2.zero_()
     g.replay()
     torch.cuda.synchronize()
     assert torch.equal(cg.z2, eager.z2)
     assert torch.equal(O1, O2)
+    assert torch.equal(K1, K2) and torch.equal(V1, V2)
+    assert torch.equal(cg.Kc, eager.Kc) and torch.equal(cg.Vc, eager.Vc)
     assert cg.status.item() == 0
 
 
