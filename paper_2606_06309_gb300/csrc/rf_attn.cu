@@ -565,13 +565,19 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       if (hasB) tc_commit(bar(C::kBarQEmpty + 1));
       continue;
     }
+    // A query tile is read by QK^T only: its buffer is released as soon as the unit's last
+    // QK^T of that tile is issued (the commit fires when it completes), so the next unit's
+    // queries, and the K/V tiles the producer queues behind them, load while this unit's last
+    // softmax and PV products still run.
     int sK, sV;
     if (!next_slot(sK)) goto fail;
     mma_qk<D>(tS[0], dQ[0], dK(sK));
     tc_commit(bar(C::kBarSFull + 0));
+    if (ntiles == 1) tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       mma_qk<D>(tS[1], dQ[1], dK(sK));
       tc_commit(bar(C::kBarSFull + 1));
+      if (ntiles == 1) tc_commit(bar(C::kBarQEmpty + 1));
     }
     tc_commit(bar(C::kBarKVEmpty + sK));
     if (!next_slot(sV)) goto fail;
@@ -582,9 +588,11 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     for (int j = 0;; ++j) {
       if (j + 1 >= ntiles) break;
       ++nj;
+      const bool last = j + 2 >= ntiles;
       if (!next_slot(sK)) goto fail;
       mma_qk<D>(tS[0], dQ[0], dK(sK));
       tc_commit(bar(C::kBarSFull + 0));
+      if (last) tc_commit(bar(C::kBarQEmpty + 0));
       if (hasB) {
         if (!wait_p(1)) goto fail;
         mma_pv<D>(tO[1], tS[1], dV(sV), j > 0);
@@ -593,6 +601,7 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       if (hasB) {
         mma_qk<D>(tS[1], dQ[1], dK(sK));
         tc_commit(bar(C::kBarSFull + 1));
+        if (last) tc_commit(bar(C::kBarQEmpty + 1));
       }
       tc_commit(bar(C::kBarKVEmpty + sK));
       if (!next_slot(sV)) goto fail;
@@ -601,12 +610,10 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     }
     if constexpr (MASKED) mbar_arrive(tl.empty(k));
     tc_commit(bar(C::kBarODone + 0));
-    tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       if (!wait_p(1)) goto fail;
       mma_pv<D>(tO[1], tS[1], dV(sV), nj > 1);
       tc_commit(bar(C::kBarODone + 1));
-      tc_commit(bar(C::kBarQEmpty + 1));
     }
     tc_commit(bar(C::kBarKVEmpty + sV));
   }
