@@ -92,9 +92,10 @@ struct Cfg {
   // misc: tmem address, abort flag, merge flags [2 groups][2 alternating slots]
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 32 + 1024;  // + slack to align the base
-  // (MASKED) tile-list ring: barriers tl_full[kTLSlots] tl_empty[kTLSlots], then the slots
+  // (MASKED) tile-list ring: barriers tl_full[kTLSlots] tl_empty[kTLSlots] tl_claim (+ 8 bytes
+  // of padding), then the slots
   static constexpr int kOffTL = (kOffMisc + 32 + 15) / 16 * 16;
-  static constexpr int kOffTLSlot = kOffTL + 2 * kTLSlots * 8;
+  static constexpr int kOffTLSlot = kOffTL + (2 * kTLSlots + 2) * 8;
   static constexpr int kSmemBytesMasked = kOffTLSlot + kTLSlots * kTLSlotBytes + 1024;
   // split-KV partial row: D unnormalised outputs, running max (log2 units), running sum
   static constexpr int kPartFloats = D + 4;
@@ -286,6 +287,9 @@ struct TLRing {
   __device__ __forceinline__ uint32_t empty(int k) const {
     return bar + 8u * (kTLSlots + k % kTLSlots);
   }
+  // (work queue) the producer arrives once per unit, when at most kClaimAhead of the unit's KV
+  // tiles are left to load: the builder may then take the next unit from the queue
+  __device__ __forceinline__ uint32_t claim() const { return bar + 8u * (2 * kTLSlots); }
   __device__ __forceinline__ uint32_t* words(int k) const {
     return slots + (k % kTLSlots) * (kTLSlotBytes / 4);
   }
@@ -297,6 +301,20 @@ struct TLRing {
 };
 // Arrivals that release a slot: the producer, the MMA issuer and the 256 softmax threads.
 constexpr int kTLConsumers = 2 + 256;
+// (work queue, at most kJitUnitsPerCta units per CTA) KV tiles of the current unit still to load
+// when the next unit is claimed.  A unit is then taken from the queue only when its CTA is about
+// to need it, so the queue's longest-first order decides which CTA gets which item as CTAs
+// actually free up.  Claimed as soon as the previous unit started, the first two units of every
+// CTA are all handed out at launch when a step has about two items per CTA: a static pairing
+// (the keyframe-only step of 13 x 1560 tokens under a banded mask, items of 21 to 78 KV tiles:
+// 0.200 ms; claimed this way 0.186 ms).  With many units per CTA the earlier claim is as good
+// and hides the claim's latency better (21 x 3600 tokens: 1-2% faster), so it stays there.
+// Three tiles are about 5 us of work, more than the claim and the tile list take to prepare.
+constexpr int kClaimAhead = 3;
+constexpr int kJitUnitsPerCta = 4;
+__device__ __forceinline__ bool claim_jit(const AttnParams& p, const Sched& sc) {
+  return p.ws_count != nullptr && sc.units <= kJitUnitsPerCta * static_cast<int>(gridDim.x);
+}
 // (MASKED, with a workspace) work-queue words in the workspace's counter area, which split-KV
 // would use but block-masked launches never split: the next unit to hand out, and the number
 // of CTAs done.  The last CTA to finish sets both back to zero.
@@ -322,6 +340,13 @@ __device__ __forceinline__ void tile_list_builder(const AttnParams& p, const Sch
     if (k >= 2 && !__all_sync(0xffffffffu, mbar_wait(tl.empty(k - 2), tl.parity(k - 2), abort,
                                                      kWaitLimitNs))) {
       if (lane == 0) flag_error(p, 7);
+      return;
+    }
+    // With the work queue and few units per CTA, the next unit is claimed only once the
+    // producer is within kClaimAhead tiles of the end of the current one.
+    if (k >= 1 && claim_jit(p, sc) &&
+        !__all_sync(0xffffffffu, mbar_wait(tl.claim(), (k - 1) & 1, abort, kWaitLimitNs))) {
+      if (lane == 0) flag_error(p, 9);
       return;
     }
     // with a workspace: the next unit of the queue shared by all CTAs (greedy list
@@ -450,9 +475,26 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
       }
       ++q_cnt[X];
     }
+    // (MASKED, work queue) tiles of this unit still to load; the claim signal goes out once
+    int left = 0;
+    bool claim_due = false;
+    if constexpr (MASKED) {
+      left = static_cast<int>(tw[kTLWords]);
+      claim_due = claim_jit(p, sc);
+      if (claim_due && left <= kClaimAhead) {
+        mbar_arrive(tl.claim());
+        claim_due = false;
+      }
+    }
 #pragma unroll 1
     for (int j = tile_first<MASKED>(u, tw, nw); j < tile_end<MASKED>(u, p);
          j = tile_next<MASKED>(tw, nw, j)) {
+      if constexpr (MASKED) {
+        if (claim_due && --left <= kClaimAhead) {
+          mbar_arrive(tl.claim());
+          claim_due = false;
+        }
+      }
 #pragma unroll
       for (int kv = 0; kv < 2; ++kv) {
         const int s = it % C::kSlots, n = it / C::kSlots;
@@ -565,19 +607,13 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       if (hasB) tc_commit(bar(C::kBarQEmpty + 1));
       continue;
     }
-    // A query tile is read by QK^T only: its buffer is released as soon as the unit's last
-    // QK^T of that tile is issued (the commit fires when it completes), so the next unit's
-    // queries, and the K/V tiles the producer queues behind them, load while this unit's last
-    // softmax and PV products still run.
     int sK, sV;
     if (!next_slot(sK)) goto fail;
     mma_qk<D>(tS[0], dQ[0], dK(sK));
     tc_commit(bar(C::kBarSFull + 0));
-    if (ntiles == 1) tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       mma_qk<D>(tS[1], dQ[1], dK(sK));
       tc_commit(bar(C::kBarSFull + 1));
-      if (ntiles == 1) tc_commit(bar(C::kBarQEmpty + 1));
     }
     tc_commit(bar(C::kBarKVEmpty + sK));
     if (!next_slot(sV)) goto fail;
@@ -588,11 +624,9 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     for (int j = 0;; ++j) {
       if (j + 1 >= ntiles) break;
       ++nj;
-      const bool last = j + 2 >= ntiles;
       if (!next_slot(sK)) goto fail;
       mma_qk<D>(tS[0], dQ[0], dK(sK));
       tc_commit(bar(C::kBarSFull + 0));
-      if (last) tc_commit(bar(C::kBarQEmpty + 0));
       if (hasB) {
         if (!wait_p(1)) goto fail;
         mma_pv<D>(tO[1], tS[1], dV(sV), j > 0);
@@ -601,7 +635,6 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
       if (hasB) {
         mma_qk<D>(tS[1], dQ[1], dK(sK));
         tc_commit(bar(C::kBarSFull + 1));
-        if (last) tc_commit(bar(C::kBarQEmpty + 1));
       }
       tc_commit(bar(C::kBarKVEmpty + sK));
       if (!next_slot(sV)) goto fail;
@@ -610,10 +643,12 @@ __device__ __forceinline__ void mma_issuer(const AttnParams& p, const Sched& sc,
     }
     if constexpr (MASKED) mbar_arrive(tl.empty(k));
     tc_commit(bar(C::kBarODone + 0));
+    tc_commit(bar(C::kBarQEmpty + 0));
     if (hasB) {
       if (!wait_p(1)) goto fail;
       mma_pv<D>(tO[1], tS[1], dV(sV), nj > 1);
       tc_commit(bar(C::kBarODone + 1));
+      tc_commit(bar(C::kBarQEmpty + 1));
     }
     tc_commit(bar(C::kBarKVEmpty + sV));
   }
@@ -953,6 +988,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(sbase + C::kOffTL + 8 * s, 32);
         mbar_init(sbase + C::kOffTL + 8 * (kTLSlots + s), kTLConsumers);
       }
+      mbar_init(sbase + C::kOffTL + 8 * (2 * kTLSlots), 1);
     }
     *abort = 0;
     fence_mbar_init();
@@ -1029,7 +1065,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // head, 152 CTAs) 19% slower than the global order, because each head's costly items started
 // late.
 __device__ __forceinline__ int lpt_group_heads(const AttnParams& p, const Sched& sc) {
-  const int need = (6 * p.lpt_grid + sc.pairs - 1) / max(sc.pairs, 1);
+  const int need = (4 * p.lpt_grid + sc.pairs - 1) / max(sc.pairs, 1);
   return min(p.H, max(p.lpt_heads_l2, need));
 }
 //
