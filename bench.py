@@ -44,6 +44,10 @@ ATTN_TRAFFIC = {
     "small": {"code_sha256_rf_attn_cu": "1dbc04774a003efa85ab66865e238dc33cd685c42928fb7b7c8cc510260628ac",
               "bytes_per_launch": 187693568 + 46976768,
               "launch": "schedule step 0 of the small workload (all 13 frames active)"},
+    "long": {"code_sha256_rf_attn_cu": "f3a9b309c12731a8ec03b6594fac9c23ea14190265eee21f174d8512fdee90ca",
+             "bytes_per_launch": 6691823165,
+             "launch": "average over the 50 launches of one trajectory of the long workload "
+                       "(21 with all 33 frames active, 29 with the 6 keyframes)"},
 }
 
 
@@ -537,6 +541,38 @@ def run_bandwidth(w, dev, peaks):
                                        "ms": round(ms1, 4)},
                      "shape": (shape or f"F={F} x E={E} fp32 (C = H*d = {D})")
                               + f", step {step}, A={nact}"}
+    # Denominators.  The measured peak is a copy (one read, one write per element); kernels that
+    # read more than they write can exceed it.  Two library kernels with other read:write mixes,
+    # timed the same way over 1 GiB fp32 operands, and the nominal HBM3e rate give context.
+    nominal = 7900.0
+    for v in res.values():
+        v["frac_of_nominal_7900"] = round(v["GB/s"] / nominal, 4)
+    n = 2 ** 28
+    xa = torch.randn(n, device=dev)
+    xb = torch.randn(n, device=dev)
+    xc = torch.empty(n, device=dev)
+    refs = {"torch_add_2_reads_1_write": (lambda: torch.add(xa, xb, out=xc), 12 * n),
+            "torch_sum_read_only": (lambda: xa.sum(), 4 * n)}
+    ref_out = {}
+    for name, (fn, nbytes) in refs.items():
+        for _ in range(3):
+            fn()
+        ts = []
+        for rep in range(7):
+            flush.fill_(rep)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        ms = statistics.median(ts)
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        ref_out[name] = {"GB/s": round(gbs, 1), "frac": round(gbs / peaks["hbm_gbs"], 4),
+                         "frac_of_nominal_7900": round(gbs / nominal, 4), "bytes": nbytes}
+    res["library_references"] = ref_out
+    del xa, xb, xc
     z2 = sets[0]["z2"]
     del sets
     # keyframe selection's inner products: proxies at latent width (where Algorithm 1 runs)
