@@ -41,11 +41,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dram__bytes_write.sum), per workload.  A figure is reported only while the kernel source
 # still has the hash it was measured with.
 ATTN_TRAFFIC = {
-    "small": {"code_sha256_rf_attn_cu": "1dbc04774a003efa85ab66865e238dc33cd685c42928fb7b7c8cc510260628ac",
-              "bytes_per_launch": 187693568 + 46976768,
-              "launch": "schedule step 0 of the small workload (all 13 frames active)"},
-    "long": {"code_sha256_rf_attn_cu": "f3a9b309c12731a8ec03b6594fac9c23ea14190265eee21f174d8512fdee90ca",
-             "bytes_per_launch": 6691823165,
+    "small": {"code_sha256_rf_attn_cu": "70d6f3611b001ebc671ab73df654848676226a2001c8d47726bc16900d557f9a",
+              "bytes_per_launch": 190560333,
+              "launch": "average over the 20 launches of one trajectory of the small workload "
+                        "(10 with all 13 frames active, 10 with the 4 keyframes)"},
+    "long": {"code_sha256_rf_attn_cu": "70d6f3611b001ebc671ab73df654848676226a2001c8d47726bc16900d557f9a",
+             "bytes_per_launch": 5118625213,
              "launch": "average over the 50 launches of one trajectory of the long workload "
                        "(21 with all 33 frames active, 29 with the 6 keyframes)"},
 }

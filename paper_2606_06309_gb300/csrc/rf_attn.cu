@@ -420,6 +420,12 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
   const int nw = (p.nkv + 31) >> 5;
   int q_cnt[2] = {0, 0};
   int it = 0;
+  // L2 priorities: a query tile is read once, a head's K/V by every unit of that head.  Marking
+  // the query loads evict-first and the K/V loads evict-last cut the DRAM reads of an
+  // all-active 33 x 3600-token launch from 8.6-10.8 GB to 7.1-9.4 GB (same box, in alternation;
+  // K/V of one head is 61 MB and is swept once per round of work items), at the same speed.
+  const uint64_t pol_q = l2_policy_evict_first();
+  const uint64_t pol_kv = l2_policy_evict_last();
   for (int k = 0;; ++k) {  // k: units so far (MASKED: tile-list ring position)
     int w;
     const uint32_t* tw = nullptr;
@@ -454,8 +460,8 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
         const int tok = p.active[a0] * p.N + (r0 - a0 * p.Np);
 #pragma unroll
         for (int hb = 0; hb < C::kHalves; ++hb)
-          tma_load_3d(dst + hb * C::kHalfBytes, tmQ128, bar(C::kBarQFull + X), hb * 64, u.h,
-                      tok);
+          tma_load_3d_hint(dst + hb * C::kHalfBytes, tmQ128, bar(C::kBarQFull + X), hb * 64,
+                           u.h, tok, pol_q);
       } else {
         // a tile across frames: gathered in boxes of 8 rows (frames are padded to 8 rows)
         int tok[BM / 8];
@@ -470,8 +476,8 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
         for (int b = 0; b < BM / 8; ++b)
 #pragma unroll
           for (int hb = 0; hb < C::kHalves; ++hb)
-            tma_load_3d(dst + hb * C::kHalfBytes + b * 1024, tmQ, bar(C::kBarQFull + X),
-                        hb * 64, u.h, tok[b]);
+            tma_load_3d_hint(dst + hb * C::kHalfBytes + b * 1024, tmQ, bar(C::kBarQFull + X),
+                             hb * 64, u.h, tok[b], pol_q);
       }
       ++q_cnt[X];
     }
@@ -506,8 +512,8 @@ __device__ __forceinline__ void producer(const CUtensorMap* tmQ, const CUtensorM
         const uint32_t dst = sKV0 + s * C::kTileBytes;
 #pragma unroll
         for (int hb = 0; hb < C::kHalves; ++hb)
-          tma_load_3d(dst + hb * C::kHalfBytes, kv ? tmV : tmK, bar(C::kBarKVFull + s), hb * 64,
-                      u.h, j * BN);
+          tma_load_3d_hint(dst + hb * C::kHalfBytes, kv ? tmV : tmK, bar(C::kBarKVFull + s),
+                           hb * 64, u.h, j * BN, pol_kv);
         ++it;
       }
     }

@@ -113,6 +113,25 @@ def test_device_calls_reject_bad_args_on_host(rf):
     assert lib.rf_attn_block_masked(*margs) == 2                      # 4097 key blocks
 
 
+def test_noalloc_rejects_bad_args_before_any_device_work(rf):
+    """rf_attn_noalloc returns rf_attn's argument errors before it looks up its scratch array
+    or enqueues the counter reset: no CUDA call happens, so this runs without a GPU."""
+    lib = rf.load()
+    P = 256
+    base = [P, None, P, P, P, 256, 256, 4, 64, 2, 128, P, P, 0.1, None, None]
+    cases = ((0, None, 1),      # null output
+             (11, None, 1),     # null active list
+             (10, 96, 2),       # head dim 96
+             (13, 0.0, 1),      # softmax scale 0
+             (5, 100, 1),       # row stride < H*d
+             (6, 260, 3),       # output row stride % 8 != 0
+             (7, 0, 1))         # no frames
+    for i, v, want in cases:
+        args = list(base)
+        args[i] = v
+        assert lib.rf_attn_noalloc(*args) == want, (i, v)
+
+
 def test_pipeline_rejects_bad_args_on_host(rf):
     """The host-fed pipeline's argument checks run before any allocation or CUDA call."""
     lib = rf.load()
