@@ -87,6 +87,8 @@ def test_device_calls_reject_bad_args_on_host(rf):
     assert lib.rf_schedule_compact(P, 0, 8, P, P, P, P, None) == 1
     assert lib.rf_project(P, P, P, P, P, 4, 6, None) == 3            # E % 4 != 0
     assert lib.rf_step(P, P, None, P, P, P, 4, 8, None) == 1
+    assert lib.rf_project(P, P, P, P, P, 4, 0, None) == 0            # E = 0: nothing to do
+    assert lib.rf_step(P, P, P, P, P, P, 4, 0, None) == 0
     args = [P, None, P, P, P, 256, 256, 4, 64, 2, 96, P, P, 0.1, None, 0, None, None]
     assert lib.rf_attn(*args) == 2                                   # d = 96 unsupported
     args[10] = 128

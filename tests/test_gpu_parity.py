@@ -128,6 +128,82 @@ def test_step_parity(cuda_lib, F, E):
     np.testing.assert_array_equal(got_new[~m], z2[1 - slot.long(), idx].double().numpy()[~m])
 
 
+def test_bandwidth_kernels_at_their_frame_limits(cuda_lib):
+    """The largest frame counts the calls accept: rf_project over 65535 frames (the grid's
+    y limit) of 4 elements; the compaction, rf_step and rf_project_kv over 4096 frames (the
+    compaction's limit, which bounds the active lists the other two read); and E = 0, which
+    launches nothing and leaves the buffers alone."""
+    rf = cuda_lib
+    g = torch.Generator().manual_seed(4096)
+    # rf_project at F = 65535
+    F, E = 65535, 4
+    z2 = torch.randn(2, F, E, generator=g)
+    slot = (torch.rand(F, generator=g) < 0.5).to(torch.uint8)
+    alpha = torch.rand(F, generator=g)
+    alpha[::7] = 1.0
+    beta = (1.0 - alpha.double()).float()
+    ctx = torch.full((F, E), SENTINEL, device=DEV)
+    rf.rf_project(ctx, z2.to(DEV), slot.to(DEV), alpha.to(DEV), beta.to(DEV), F, E)
+    torch.cuda.synchronize()
+    idx = torch.arange(F)
+    cur, prev = z2[slot.long(), idx], z2[1 - slot.long(), idx]
+    want = oracle.project(prev, cur, alpha.double().numpy())
+    terms = np.abs(beta.double().numpy()[:, None] * prev.double().numpy()) + \
+        np.abs(alpha.double().numpy()[:, None] * cur.double().numpy())
+    assert _rel_err(ctx.cpu().double().numpy(), want, terms) <= 1e-5
+    # compaction, rf_step and rf_project_kv at F = 4096
+    F, N, D, E = 4096, 1, 8, 8
+    mask = (torch.rand(F, generator=g) < 0.3).to(torch.uint8)
+    mask[-1] = 1
+    act = torch.full((F,), -1, dtype=torch.int32, device=DEV)
+    skp = torch.full((F,), -1, dtype=torch.int32, device=DEV)
+    cnt = torch.zeros(2, dtype=torch.int32, device=DEV)
+    rf.rf_schedule_compact(mask.to(DEV), F, N, act, skp, None, cnt)
+    z2 = torch.randn(2, F, E, generator=g)
+    v = torch.randn(F, E, generator=g)
+    slot = (torch.rand(F, generator=g) < 0.5).to(torch.uint8)
+    dt = -torch.rand(F, generator=g)
+    d_z2 = z2.to(DEV)
+    rf.rf_step(d_z2, slot.to(DEV), v.to(DEV), dt.to(DEV), act, cnt, F, E)
+    torch.cuda.synchronize()
+    idx = torch.arange(F)
+    cur = z2[slot.long(), idx]
+    m = mask.numpy().astype(bool)
+    got = d_z2.cpu()[1 - slot.long(), idx].double().numpy()
+    want = oracle.euler(cur, v, dt.double().numpy())
+    terms = np.abs(cur.double().numpy()) + np.abs(dt.double().numpy()[:, None] * v.double().numpy())
+    assert _rel_err(got[m], want[m], terms[m]) <= 1e-5
+    np.testing.assert_array_equal(got[~m], z2[1 - slot.long(), idx].double().numpy()[~m])
+    K = torch.randn(F * N, D, generator=g).to(torch.bfloat16)
+    V = torch.randn(F * N, D, generator=g).to(torch.bfloat16)
+    Kc = torch.randn(2, F, N, D, generator=g).to(torch.bfloat16)
+    Vc = torch.randn(2, F, N, D, generator=g).to(torch.bfloat16)
+    al = torch.rand(F, generator=g)
+    al[m] = 1.0
+    be = (1.0 - al.double()).float()
+    dK, dV, dKc, dVc = (x.to(DEV) for x in (K, V, Kc, Vc))
+    rf.rf_project_kv(dK, dV, D, dKc, dVc, slot.to(DEV), al.to(DEV), be.to(DEV), act, skp, cnt,
+                     F, N, D)
+    torch.cuda.synchronize()
+    for X, c, dX, dc in ((K, Kc, dK, dKc), (V, Vc, dV, dVc)):
+        want, want_c = oracle.project_kv_cache(X.view(F, N, D), c, slot.numpy(), al.numpy(),
+                                               mask.numpy())
+        got = dX.cpu().double().view(F, N, D).numpy()
+        c0 = c.double().numpy()
+        sl = slot.numpy().astype(np.int64)
+        terms = (np.abs(be.double().numpy())[:, None, None] * np.abs(c0[1 - sl, idx])
+                 + np.abs(al.double().numpy())[:, None, None] * np.abs(c0[sl, idx]))
+        assert (np.abs(got[~m] - want[~m]) <= 2.0 ** -8 * terms[~m] + 1e-30).all()
+        np.testing.assert_array_equal(got[m], X.view(F, N, D).double().numpy()[m])
+        np.testing.assert_array_equal(dc.cpu().double().numpy(), want_c)
+    # E = 0: nothing is launched, nothing is written
+    before = d_z2.clone()
+    rf.rf_step(d_z2, slot.to(DEV), v.to(DEV), dt.to(DEV), act, cnt, F, 0)
+    rf.rf_project(ctx, d_z2, slot.to(DEV), al.to(DEV), be.to(DEV), F, 0)
+    torch.cuda.synchronize()
+    assert torch.equal(d_z2, before)
+
+
 # ---------------------------------------------------------------------------
 # rf_attn
 # ---------------------------------------------------------------------------
@@ -214,6 +290,8 @@ def test_attn_tiny_every_step(cuda_lib):
     (64, 1, 2, 128, [1, 1, 0, 1] * 16),   # N = 1: seven padded rows per frame
     (3, 4096, 1, 128, [1, 0, 1]),         # frames of whole tiles (one 128-row box each)
     (2, 1, 1, 64, [1, 1]),                # two tokens in all
+    (1, 8, 1024, 64, [1]),                # 1024 heads of one 8-row tile: many short items
+    (2, 4, 300, 128, [0, 1]),             # 300 heads, one active frame of 4 tokens
 ])
 def test_attn_ragged_shapes(cuda_lib, F, N, H, d, mask):
     rf = cuda_lib
