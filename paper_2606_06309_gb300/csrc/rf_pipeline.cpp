@@ -211,7 +211,6 @@ extern "C" rf_status rf_pipeline_step(rf_pipeline* p, int s, const void* h_Q, co
     f = g;
   }
   int64_t active_bytes = 0;
-  // host -> device
   // host -> device: the fresh Q, K and V rows of the active frames, and the velocity
   if (!first_use) CUDA_TRY(cudaStreamWaitEvent(p->h2d, B.consumed, 0), "rf_pipeline h2d wait");
   for (const auto& r : runs) {
