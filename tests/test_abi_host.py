@@ -232,3 +232,17 @@ def test_keyframe_select_scene_starts(rf):
     assert np.flatnonzero(got).tolist() == [0, 4, 9, 13, 17]
     with pytest.raises(rf.RFError):
         rf.rf_keyframe_select(np.zeros((3, 3)), 2, 0.5, 0.0, 1, 1)   # zero-norm frames
+
+
+def test_bench_traffic_figures_belong_to_the_current_kernel():
+    """bench.py reports roofline.traffic only while rf_attn.cu (without comments) hashes to the
+    key its ncu capture was taken with; the committed figures are those of the current kernel."""
+    import os
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    import bench
+    sha = bench._code_sha(os.path.join(root, "paper_2606_06309_gb300", "csrc", "rf_attn.cu"))
+    for name, entry in bench.ATTN_TRAFFIC.items():
+        assert entry["code_sha256_rf_attn_cu"] == sha, name
+        assert entry["bytes_per_launch"] > 0
