@@ -444,6 +444,29 @@ def test_attn_small_every_row_of_two_heads(cuda_lib, s):
             Lref, f"small s={s} every row, heads {heads}")
 
 
+@pytest.mark.parametrize("name", ["large", "long"])
+def test_attn_every_row_of_two_heads_keyframe_step(cuda_lib, name):
+    """Every active row of the first and last head on the keyframe-only step of the 21 and
+    33 x 3600-token workloads (6 keyframes: 21600 query rows against all keys), in the
+    benchmark's launch configuration, against the fp64 oracle.  The large workload's tokens
+    with std 2 give the rows that a few keys dominate."""
+    rf = cuda_lib
+    w = wl.get(name)
+    Q, K, V = wl.qkv(w, device=DEV)
+    p = _plan(rf, w)
+    s = int(p["mask"].sum(axis=1).argmin())
+    mask = p["mask"][s]
+    O, L = _run_attn(rf, Q, K, V, w.F, w.N, mask, w.softmax_scale)
+    rows = _active_rows(mask, w.N)
+    heads = [0, w.H - 1]
+    hq = torch.tensor(heads, device=DEV)
+    Qs, Ks, Vs = (x.index_select(1, hq).cpu() for x in (Q, K, V))
+    Oref, Lref = oracle.attention(Qs, Ks, Vs, rows, w.softmax_scale)
+    compare(O.index_select(1, hq).cpu().float()[rows].numpy(), Oref,
+            L.index_select(0, hq).cpu()[:, rows].numpy(), Lref,
+            f"{name} step {s} every row, heads {heads}")
+
+
 # ---------------------------------------------------------------------------
 # Whole trajectory: compaction + projection + attention + Euler step, S steps
 # ---------------------------------------------------------------------------
